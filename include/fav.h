@@ -1,0 +1,133 @@
+/*
+ * fav.h -- libfav: exact fused attention forward on one NVIDIA GB300 (sm_103a).
+ *
+ * The operation is scaled dot-product attention as defined in the FlashAttention-V paper
+ * (Background section: Attention(Q,K,V) = softmax(Q K^T / sqrt(D)) V), evaluated with the
+ * tiled online softmax of its Method section (Algorithm "ggml-vec FlashAttention in
+ * llama.cpp" and Algorithm "FlashAttention-V for VL > D"), for multi-head, grouped-query and
+ * multi-query attention (Method section on GQA), prefill (Nq = Nkv) and decode (Nq = 1).
+ *
+ * Conventions shared by every entry point below
+ * ---------------------------------------------
+ *  Layouts   q, o : [B, Hq,  Nq,  D]  contiguous row-major, element type `dtype`
+ *            k, v : [B, Hkv, Nkv, D]  contiguous row-major, element type `dtype`
+ *            lse  : [B, Hq,  Nq]      contiguous fp32, natural-log log-sum-exp of the scaled
+ *                                      scores of each query row (may be NULL: not written)
+ *  Heads     query head h reads K/V head h / (Hq / Hkv): consecutive query heads share.
+ *  Causal    bottom-right aligned: query i sees keys j <= Nkv - Nq + i (needs Nq <= Nkv).
+ *  Scale     applied to Q.K before the softmax; callers pass 1/sqrt(D).  Must be finite, > 0.
+ *  Precision fp32 I/O: exact fp32 arithmetic.  fp16 / bf16 I/O: fp32 accumulation; on the
+ *            tensor-core paths the softmax weights P are rounded (to nearest even) to the
+ *            I/O type before the P.V product (the CUDA-core path keeps them in fp32);
+ *            O is rounded to the I/O type once, at the end.
+ *  Ownership every pointer is caller-owned; the library never frees or retains it.
+ *  Errors    arguments are validated before anything is launched, so an error status
+ *            leaves o and lse untouched.  There is no CPU fallback.
+ */
+#ifndef FAV_H
+#define FAV_H
+
+#if defined(__GNUC__)
+#define FAV_API __attribute__((visibility("default")))
+#else
+#define FAV_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum { FAV_F32 = 0, FAV_F16 = 1, FAV_BF16 = 2 } fav_dtype;
+
+typedef enum {
+    FAV_OK = 0,
+    FAV_ERR_INVALID_ARG = 1,    /* null or misaligned pointer, bad size, Hq % Hkv != 0, ...   */
+    FAV_ERR_UNSUPPORTED = 2,    /* valid attention problem that no kernel here implements     */
+    FAV_ERR_CUDA = 3,           /* a CUDA runtime call or kernel launch failed                */
+    FAV_ERR_NO_MEMORY = 4,      /* the internal workspace could not be allocated              */
+    FAV_ERR_DEVICE_TIMEOUT = 5  /* a bounded wait inside a kernel ran out (see below)         */
+} fav_status;
+
+/* Kernel families (for fav_set_path / fav_last_path). */
+typedef enum {
+    FAV_PATH_AUTO = 0,    /* choose by dtype and shape (default)                               */
+    FAV_PATH_SIMT = 1,    /* generic CUDA-core kernel, any dtype, D % 8 == 0 (D % 4 for fp32),
+                             D <= 256; exact fp32 arithmetic for fp32 I/O                     */
+    FAV_PATH_DECODE = 2,  /* split-KV decode kernel + log-sum-exp combine; fp16/bf16,
+                             D in {64, 128}, Nq * (Hq / Hkv) <= 64 query rows per KV head
+                             (taken in blocks of 16 MMA rows; auto-chosen when <= 16)         */
+    FAV_PATH_PREFILL = 3  /* tcgen05 / TMEM / TMA prefill kernel; fp16/bf16, D in {64, 128}   */
+} fav_path;
+
+/*
+ * fav_forward -- O = softmax(scale * Q K^T [masked]) V and LSE, asynchronously on `stream`.
+ *
+ *  q, k, v   device pointers (layouts above), 16-byte aligned
+ *  o         device pointer, [B, Hq, Nq, D] of `dtype`, 16-byte aligned
+ *  lse       device pointer [B, Hq, Nq] fp32 (4-byte aligned), or NULL
+ *  B..D      sizes, all > 0; Hq % Hkv == 0; causal requires Nq <= Nkv
+ *  scale     finite and > 0
+ *  causal    0 or 1
+ *  dtype     FAV_F32, FAV_F16 or FAV_BF16 (the type of q, k, v and o)
+ *  stream    a cudaStream_t (NULL = the legacy default stream)
+ *
+ * Decode-shaped calls (small Nq * Hq / Hkv) split the key range over thread blocks and merge
+ * the partial results with a log-sum-exp combine (associativity of the online softmax); the
+ * partials live in an internal device workspace that grows on demand (cudaMallocAsync on
+ * `stream`) and is kept until fav_release_workspace().  FAV_ERR_NO_MEMORY if that fails.
+ * Returns FAV_OK once the kernels are enqueued; it does not synchronise.
+ */
+FAV_API fav_status fav_forward(const void *q, const void *k, const void *v, void *o, float *lse,
+                       int B, int Hq, int Hkv, int Nq, int Nkv, int D,
+                       float scale, int causal, fav_dtype dtype, void *stream);
+
+/*
+ * fav_forward_host -- the same operation on HOST buffers (end-to-end call).
+ *
+ * Copies q, k, v (host, ideally pinned) to internal device buffers, runs fav_forward on
+ * `stream`, copies o and lse (lse may be NULL) back to the host and synchronises `stream`.
+ * The device buffers grow on demand and are kept until fav_release_workspace().
+ * Host pointers need no alignment.  Same argument rules and statuses as fav_forward.
+ */
+FAV_API fav_status fav_forward_host(const void *q, const void *k, const void *v, void *o, float *lse,
+                            int B, int Hq, int Hkv, int Nq, int Nkv, int D,
+                            float scale, int causal, fav_dtype dtype, void *stream);
+
+/* A short English description of a status code (static storage, never NULL). */
+FAV_API const char *fav_status_string(fav_status s);
+
+/*
+ * fav_get_last_device_status -- synchronises the device, then reports and clears the status
+ * word that kernels set when one of their bounded waits (on an mbarrier) gave up:
+ * FAV_OK or FAV_ERR_DEVICE_TIMEOUT.  FAV_ERR_CUDA if the device could not be queried.
+ */
+FAV_API fav_status fav_get_last_device_status(void);
+
+/* Frees the internal workspace and host-call buffers of the current device (synchronises). */
+FAV_API void fav_release_workspace(void);
+
+/*
+ * fav_set_path -- process-wide override of the kernel family (FAV_PATH_AUTO restores the
+ * default choice).  A forced path that cannot run a given call makes fav_forward return
+ * FAV_ERR_UNSUPPORTED.  Intended for tests and measurements.
+ */
+FAV_API fav_status fav_set_path(fav_path p);
+
+/* The kernel family used by the last successful fav_forward call of this process. */
+FAV_API fav_path fav_last_path(void);
+
+/*
+ * fav_set_decode_splits -- process-wide number of key-range splits for the decode path
+ * (0 = automatic, from the problem size and the SM count).  Values are clamped to the number
+ * of key tiles.  FAV_ERR_INVALID_ARG for n < 0 or n > 4096.
+ */
+FAV_API fav_status fav_set_decode_splits(int n);
+
+/* The split count the last decode-path fav_forward call used (0 if none ran yet). */
+FAV_API int fav_last_decode_splits(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FAV_H */

@@ -1,0 +1,155 @@
+"""libfav Python binding: argument marshalling onto the C ABI declared in include/fav.h.
+
+Every step of the attention forward runs in the CUDA kernels of ``libfav.so``; this module
+only turns torch CUDA tensors into pointers, sizes and the current stream.  There is no
+CPU fallback: without the built library every call raises.
+"""
+import ctypes
+import os
+
+__all__ = ["forward", "forward_host", "set_path", "last_path", "set_decode_splits",
+           "last_decode_splits", "device_status", "release_workspace", "library_path",
+           "FavError", "F32", "F16", "BF16", "PATH_AUTO", "PATH_SIMT", "PATH_DECODE",
+           "PATH_PREFILL"]
+
+F32, F16, BF16 = 0, 1, 2
+PATH_AUTO, PATH_SIMT, PATH_DECODE, PATH_PREFILL = 0, 1, 2, 3
+PATH_NAMES = {PATH_AUTO: "auto", PATH_SIMT: "simt", PATH_DECODE: "decode",
+              PATH_PREFILL: "prefill"}
+STATUS_NAMES = {0: "FAV_OK", 1: "FAV_ERR_INVALID_ARG", 2: "FAV_ERR_UNSUPPORTED",
+                3: "FAV_ERR_CUDA", 4: "FAV_ERR_NO_MEMORY", 5: "FAV_ERR_DEVICE_TIMEOUT"}
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libfav.so")
+_lib = None
+
+
+class FavError(RuntimeError):
+    def __init__(self, status, msg=""):
+        self.status = status
+        super().__init__("%s%s" % (STATUS_NAMES.get(status, status), (": " + msg) if msg else ""))
+
+
+def library_path():
+    return _LIB_PATH
+
+
+def lib():
+    """The loaded libfav.so (raises if it was not built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError("libfav.so is not built; run __graft_entry__.build() "
+                               "(or python paper_2608_18656_gb300/build.py)")
+        L = ctypes.CDLL(_LIB_PATH)
+        vp, i = ctypes.c_void_p, ctypes.c_int
+        sig = [vp, vp, vp, vp, vp, i, i, i, i, i, i, ctypes.c_float, i, i, vp]
+        for fn in ("fav_forward", "fav_forward_host"):
+            getattr(L, fn).argtypes = sig
+            getattr(L, fn).restype = i
+        L.fav_status_string.argtypes = [i]
+        L.fav_status_string.restype = ctypes.c_char_p
+        L.fav_get_last_device_status.argtypes = []
+        L.fav_get_last_device_status.restype = i
+        L.fav_release_workspace.argtypes = []
+        L.fav_release_workspace.restype = None
+        L.fav_set_path.argtypes = [i]
+        L.fav_set_path.restype = i
+        L.fav_last_path.argtypes = []
+        L.fav_last_path.restype = i
+        L.fav_set_decode_splits.argtypes = [i]
+        L.fav_set_decode_splits.restype = i
+        L.fav_last_decode_splits.argtypes = []
+        L.fav_last_decode_splits.restype = i
+        _lib = L
+    return _lib
+
+
+def _check(st):
+    if st != 0:
+        raise FavError(st, lib().fav_status_string(st).decode())
+
+
+def _dtype_code(t):
+    import torch
+    codes = {torch.float32: F32, torch.float16: F16, torch.bfloat16: BF16}
+    if t.dtype not in codes:
+        raise TypeError("unsupported dtype %s" % t.dtype)
+    return codes[t.dtype]
+
+
+def forward(q, k, v, causal=False, scale=None, return_lse=True, out=None, lse_out=None,
+            stream=None):
+    """Attention forward on torch CUDA tensors q [B,Hq,Nq,D], k/v [B,Hkv,Nkv,D].
+
+    Returns (o, lse) with lse [B,Hq,Nq] fp32 (None if return_lse is False).  Runs on the
+    current torch stream unless ``stream`` (a torch.cuda.Stream) is given.
+    """
+    import torch
+    for t in (q, k, v):
+        if not t.is_cuda:
+            raise ValueError("tensors must live on a CUDA device")
+        if not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+    if k.dtype != q.dtype or v.dtype != q.dtype:
+        raise TypeError("q, k and v must share a dtype")
+    B, Hq, Nq, D = q.shape
+    Bk, Hkv, Nkv, Dk = k.shape
+    if tuple(v.shape) != tuple(k.shape) or Bk != B or Dk != D:
+        raise ValueError("shape mismatch between q, k and v")
+    if scale is None:
+        import numpy as np
+        scale = float(np.float32(1.0 / np.sqrt(D)))
+    o = out if out is not None else torch.empty_like(q)
+    lse = None
+    if return_lse:
+        lse = lse_out if lse_out is not None else torch.empty((B, Hq, Nq), device=q.device,
+                                                              dtype=torch.float32)
+    s = stream if stream is not None else torch.cuda.current_stream(q.device)
+    with torch.cuda.device(q.device):
+        st = lib().fav_forward(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(),
+                               lse.data_ptr() if lse is not None else None, B, Hq, Hkv, Nq,
+                               Nkv, D, float(scale), int(bool(causal)), _dtype_code(q),
+                               s.cuda_stream)
+    _check(st)
+    return o, lse
+
+
+def forward_host(q, k, v, o, lse, B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype, stream=0):
+    """End-to-end call on host buffers (numpy arrays or raw addresses); synchronises."""
+    def addr(a):
+        if a is None:
+            return None
+        if isinstance(a, int):
+            return a
+        if hasattr(a, "ctypes"):
+            return a.ctypes.data
+        return a.data_ptr()
+    st = lib().fav_forward_host(addr(q), addr(k), addr(v), addr(o), addr(lse), B, Hq, Hkv, Nq,
+                                Nkv, D, float(scale), int(bool(causal)), int(dtype), stream)
+    _check(st)
+
+
+def set_path(path):
+    _check(lib().fav_set_path(int(path)))
+
+
+def last_path():
+    return lib().fav_last_path()
+
+
+def set_decode_splits(n):
+    _check(lib().fav_set_decode_splits(int(n)))
+
+
+def last_decode_splits():
+    return lib().fav_last_decode_splits()
+
+
+def device_status():
+    """Synchronises; returns and clears the kernels' bounded-wait status (0 = ok)."""
+    return lib().fav_get_last_device_status()
+
+
+def release_workspace():
+    lib().fav_release_workspace()

@@ -1,0 +1,311 @@
+// fav_api.cu -- the C ABI of libfav (declared in include/fav.h): argument validation,
+// kernel-family dispatch, the internal split-KV workspace, host-buffer calls, tensor maps.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <stdlib.h>
+
+#include <algorithm>
+#include <atomic>
+#include <mutex>
+
+#include "fav_internal.h"
+
+// Status word written by kernels whose bounded waits gave up (FAV_ERR_DEVICE_TIMEOUT).
+__device__ int g_fav_device_status;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceState {
+    bool init = false;
+    int *status = nullptr;     // device address of g_fav_device_status
+    int num_sms = 0;
+    void *ws = nullptr;        // split-KV partials
+    size_t ws_bytes = 0;
+    void *hbuf = nullptr;      // device copies for fav_forward_host
+    size_t hbuf_bytes = 0;
+};
+
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+std::atomic<int> g_path{FAV_PATH_AUTO};
+std::atomic<int> g_last_path{FAV_PATH_AUTO};
+std::atomic<int> g_splits{0};
+std::atomic<int> g_last_splits{0};
+
+fav_status device_state(DeviceState **out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FAV_ERR_CUDA;
+    DeviceState &d = g_dev[dev];
+    if (!d.init) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_fav_device_status) != cudaSuccess) return FAV_ERR_CUDA;
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return FAV_ERR_CUDA;
+        d.status = static_cast<int *>(p);
+        d.num_sms = sms;
+        d.init = true;
+    }
+    *out = &d;
+    return FAV_OK;
+}
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+fav_status validate_shape(int B, int Hq, int Hkv, int Nq, int Nkv, int D, float scale,
+                          int causal, fav_dtype dtype) {
+    if (B <= 0 || Hq <= 0 || Hkv <= 0 || Nq <= 0 || Nkv <= 0 || D <= 0) return FAV_ERR_INVALID_ARG;
+    if (Hq % Hkv != 0) return FAV_ERR_INVALID_ARG;
+    if (causal != 0 && causal != 1) return FAV_ERR_INVALID_ARG;
+    if (causal && Nq > Nkv) return FAV_ERR_INVALID_ARG;
+    if (!(scale > 0.f) || !isfinite(scale)) return FAV_ERR_INVALID_ARG;
+    if (dtype != FAV_F32 && dtype != FAV_F16 && dtype != FAV_BF16) return FAV_ERR_INVALID_ARG;
+    const int es = dtype == FAV_F32 ? 4 : 2;
+    if ((D * es) % 16 != 0) return FAV_ERR_UNSUPPORTED;        // rows must stay 16-byte aligned
+    // Element counts must fit the kernels' 32-bit grid and 64-bit index arithmetic.
+    const long long rows = (long long)B * Hq * Nq;
+    if (rows > (1LL << 40) || (long long)B * Hkv * Nkv > (1LL << 40)) return FAV_ERR_UNSUPPORTED;
+    return FAV_OK;
+}
+
+FavArgs make_args(const void *q, const void *k, const void *v, void *o, float *lse, int B, int Hq,
+                  int Hkv, int Nq, int Nkv, int D, float scale, int causal, fav_dtype dtype) {
+    FavArgs a;
+    a.q = q; a.k = k; a.v = v; a.o = o; a.lse = lse;
+    a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.Nq = Nq; a.Nkv = Nkv; a.D = D;
+    a.scale = scale; a.causal = causal; a.dtype = dtype;
+    a.dev_status = nullptr;
+    a.num_sms = 0;
+    return a;
+}
+
+bool decode_shaped(const FavArgs &a) {
+    return (long long)a.Nq * (a.Hq / a.Hkv) <= 16;
+}
+
+// Chooses the kernel family for a validated call; FAV_PATH_AUTO if none can run it.
+fav_path choose_path(const FavArgs &a) {
+    const int forced = g_path.load();
+    switch (forced) {
+    case FAV_PATH_SIMT: return fav_simt_supported(a) ? FAV_PATH_SIMT : FAV_PATH_AUTO;
+    case FAV_PATH_DECODE: return fav_decode_supported(a) ? FAV_PATH_DECODE : FAV_PATH_AUTO;
+    case FAV_PATH_PREFILL: return fav_prefill_supported(a) ? FAV_PATH_PREFILL : FAV_PATH_AUTO;
+    default: break;
+    }
+    if (a.dtype != FAV_F32) {
+        if (decode_shaped(a) && fav_decode_supported(a)) return FAV_PATH_DECODE;
+        if (fav_prefill_supported(a)) return FAV_PATH_PREFILL;
+        if (fav_decode_supported(a)) return FAV_PATH_DECODE;
+    }
+    if (fav_simt_supported(a)) return FAV_PATH_SIMT;
+    return FAV_PATH_AUTO;
+}
+
+fav_status ensure_buffer(void **ptr, size_t *have, size_t need, cudaStream_t s) {
+    if (need <= *have) return FAV_OK;
+    if (*ptr) {
+        cudaFreeAsync(*ptr, s);
+        *ptr = nullptr;
+        *have = 0;
+    }
+    void *p = nullptr;
+    if (cudaMallocAsync(&p, need, s) != cudaSuccess) {
+        cudaGetLastError();
+        return FAV_ERR_NO_MEMORY;
+    }
+    *ptr = p;
+    *have = need;
+    return FAV_OK;
+}
+
+fav_status forward_impl(const FavArgs &in, cudaStream_t stream) {
+    DeviceState *ds = nullptr;
+    fav_status st = device_state(&ds);
+    if (st != FAV_OK) return st;
+    FavArgs a = in;
+    a.dev_status = ds->status;
+    a.num_sms = ds->num_sms;
+    const fav_path path = choose_path(a);
+    if (path == FAV_PATH_AUTO) return FAV_ERR_UNSUPPORTED;
+    cudaGetLastError();   // a stale error from elsewhere must not be reported as ours
+    switch (path) {
+    case FAV_PATH_SIMT:
+        st = fav_launch_simt(a, stream);
+        break;
+    case FAV_PATH_PREFILL:
+        st = fav_launch_prefill(a, stream);
+        break;
+    case FAV_PATH_DECODE: {
+        const int n_tiles = fav_decode_num_tiles(a);
+        int splits = g_splits.load();
+        if (splits <= 0) splits = fav_decode_auto_splits(a);
+        splits = std::max(1, std::min(splits, n_tiles));
+        const int tps = (n_tiles + splits - 1) / splits;
+        splits = (n_tiles + tps - 1) / tps;
+        void *ws = nullptr;
+        const size_t need = fav_decode_workspace_bytes(a, splits);
+        if (need) {
+            std::lock_guard<std::mutex> lk(g_mu);
+            st = ensure_buffer(&ds->ws, &ds->ws_bytes, need, stream);
+            ws = ds->ws;
+        }
+        if (st == FAV_OK) st = fav_launch_decode(a, splits, ws, stream);
+        if (st == FAV_OK) g_last_splits.store(splits);
+        break;
+    }
+    default:
+        st = FAV_ERR_UNSUPPORTED;
+    }
+    if (st == FAV_OK) g_last_path.store(path);
+    return st;
+}
+
+}  // namespace
+
+bool fav_debug_sync(const char *what, cudaStream_t s) {
+    static const bool on = [] {
+        const char *e = getenv("FAV_DEBUG_SYNC");
+        return e && e[0] == '1';
+    }();
+    if (!on) return false;
+    const cudaError_t e = cudaStreamSynchronize(s);
+    fprintf(stderr, "[fav debug] %s: %s\n", what, cudaGetErrorString(e));
+    return e != cudaSuccess;
+}
+
+fav_status fav_make_tmap_3d(void *tmap, const void *base, int D, int rows, int outer, int box_rows) {
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    });
+    if (!encode) return FAV_ERR_CUDA;
+    const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)outer};
+    const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)rows * D * 2};
+    const cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = encode(reinterpret_cast<CUtensorMap *>(tmap), CU_TENSOR_MAP_DATA_TYPE_UINT16, 3,
+                        const_cast<void *>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? FAV_OK : FAV_ERR_CUDA;
+}
+
+extern "C" {
+
+fav_status fav_forward(const void *q, const void *k, const void *v, void *o, float *lse, int B,
+                       int Hq, int Hkv, int Nq, int Nkv, int D, float scale, int causal,
+                       fav_dtype dtype, void *stream) {
+    if (!q || !k || !v || !o) return FAV_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(o, 16))
+        return FAV_ERR_INVALID_ARG;
+    if (lse && !aligned(lse, 4)) return FAV_ERR_INVALID_ARG;
+    fav_status st = validate_shape(B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    if (st != FAV_OK) return st;
+    const FavArgs a = make_args(q, k, v, o, lse, B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    return forward_impl(a, static_cast<cudaStream_t>(stream));
+}
+
+fav_status fav_forward_host(const void *q, const void *k, const void *v, void *o, float *lse,
+                            int B, int Hq, int Hkv, int Nq, int Nkv, int D, float scale,
+                            int causal, fav_dtype dtype, void *stream) {
+    if (!q || !k || !v || !o) return FAV_ERR_INVALID_ARG;
+    fav_status st = validate_shape(B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    if (st != FAV_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DeviceState *ds = nullptr;
+    st = device_state(&ds);
+    if (st != FAV_OK) return st;
+    const size_t es = dtype == FAV_F32 ? 4 : 2;
+    auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+    const size_t qb = (size_t)B * Hq * Nq * D * es;
+    const size_t kb = (size_t)B * Hkv * Nkv * D * es;
+    const size_t lb = (size_t)B * Hq * Nq * sizeof(float);
+    const size_t need = up(qb) * 2 + up(kb) * 2 + up(lb);
+    uint8_t *base = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        st = ensure_buffer(&ds->hbuf, &ds->hbuf_bytes, need, s);
+        base = static_cast<uint8_t *>(ds->hbuf);
+    }
+    if (st != FAV_OK) return st;
+    uint8_t *dq = base, *dk = dq + up(qb), *dv = dk + up(kb), *dout = dv + up(kb);
+    float *dl = reinterpret_cast<float *>(dout + up(qb));
+    if (cudaMemcpyAsync(dq, q, qb, cudaMemcpyHostToDevice, s) != cudaSuccess ||
+        cudaMemcpyAsync(dk, k, kb, cudaMemcpyHostToDevice, s) != cudaSuccess ||
+        cudaMemcpyAsync(dv, v, kb, cudaMemcpyHostToDevice, s) != cudaSuccess)
+        return FAV_ERR_CUDA;
+    const FavArgs a = make_args(dq, dk, dv, dout, lse ? dl : nullptr, B, Hq, Hkv, Nq, Nkv, D,
+                                scale, causal, dtype);
+    st = forward_impl(a, s);
+    if (st != FAV_OK) return st;
+    if (cudaMemcpyAsync(o, dout, qb, cudaMemcpyDeviceToHost, s) != cudaSuccess) return FAV_ERR_CUDA;
+    if (lse && cudaMemcpyAsync(lse, dl, lb, cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return FAV_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return FAV_ERR_CUDA;
+    return FAV_OK;
+}
+
+const char *fav_status_string(fav_status s) {
+    switch (s) {
+    case FAV_OK: return "ok";
+    case FAV_ERR_INVALID_ARG: return "invalid argument";
+    case FAV_ERR_UNSUPPORTED: return "unsupported problem for the available kernels";
+    case FAV_ERR_CUDA: return "CUDA runtime error";
+    case FAV_ERR_NO_MEMORY: return "workspace allocation failed";
+    case FAV_ERR_DEVICE_TIMEOUT: return "a bounded device wait timed out";
+    }
+    return "unknown status";
+}
+
+fav_status fav_get_last_device_status(void) {
+    DeviceState *ds = nullptr;
+    if (device_state(&ds) != FAV_OK) return FAV_ERR_CUDA;
+    if (cudaDeviceSynchronize() != cudaSuccess) return FAV_ERR_CUDA;
+    int v = 0;
+    const int zero = 0;
+    if (cudaMemcpyFromSymbol(&v, g_fav_device_status, sizeof(int)) != cudaSuccess) return FAV_ERR_CUDA;
+    if (cudaMemcpyToSymbol(g_fav_device_status, &zero, sizeof(int)) != cudaSuccess) return FAV_ERR_CUDA;
+    return v == 0 ? FAV_OK : static_cast<fav_status>(v);
+}
+
+void fav_release_workspace(void) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return;
+    std::lock_guard<std::mutex> lk(g_mu);
+    DeviceState &d = g_dev[dev];
+    cudaDeviceSynchronize();
+    if (d.ws) cudaFree(d.ws);
+    if (d.hbuf) cudaFree(d.hbuf);
+    d.ws = d.hbuf = nullptr;
+    d.ws_bytes = d.hbuf_bytes = 0;
+}
+
+fav_status fav_set_path(fav_path p) {
+    if (p < FAV_PATH_AUTO || p > FAV_PATH_PREFILL) return FAV_ERR_INVALID_ARG;
+    g_path.store(p);
+    return FAV_OK;
+}
+
+fav_path fav_last_path(void) { return static_cast<fav_path>(g_last_path.load()); }
+
+fav_status fav_set_decode_splits(int n) {
+    if (n < 0 || n > 4096) return FAV_ERR_INVALID_ARG;
+    g_splits.store(n);
+    return FAV_OK;
+}
+
+int fav_last_decode_splits(void) { return g_last_splits.load(); }
+
+}  // extern "C"

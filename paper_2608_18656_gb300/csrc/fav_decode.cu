@@ -1,0 +1,453 @@
+// fav_decode.cu -- bandwidth-bound decode attention: split-KV over thread blocks, the query
+// heads of one GQA/MQA group packed as MMA rows, and a log-sum-exp combine of the splits.
+//
+// Method (paper, Method section): the decode stage is attention of a 1 x D query per head
+// against the whole N x D key/value cache; heads that share a KV head read it once
+// (GQA support: "K and V are loaded once and reused across shared attention heads").  On this
+// GPU the roles of the paper's vector register packing are taken by tensor-core MMA rows:
+// the Nq * G query rows that read KV head g form the M = 16 rows of an m16n8k16 MMA, so one
+// pass over a K/V tile serves the whole group.
+//
+// Work decomposition: grid = (split, b * Hkv + g, 16-row chunk).  Each block streams its
+// range of 32-key tiles through a ring of shared-memory stages filled by TMA (one producer
+// warp, 128-byte swizzle), and four consumer warps take every fourth tile:
+//   S = Q K^T (mma.sync, fp32 accumulate)  ->  mask (key >= Nkv; causal, bottom-right)
+//   -> online softmax in the exp2 domain (running max, rescale of O and l)
+//   -> O += P V with P rounded to the I/O type.
+// The four warp states are merged through shared memory; with one split the block writes O
+// and LSE directly, otherwise it writes the fp32 partial (O_s, lse_s) of its key range and
+// fav_combine_kernel merges them: L = logsumexp_s lse_s, O = sum_s exp(lse_s - L) O_s
+// (associativity of the online softmax of the paper's Algorithm "ggml-vec FlashAttention").
+#include <cuda.h>
+#include <math.h>
+
+#include "fav_device.cuh"
+#include "fav_internal.h"
+
+namespace {
+
+constexpr int TK = 32;            // keys per tile
+constexpr int kConsumers = 4;     // consumer warps
+constexpr int kThreads = (kConsumers + 1) * 32;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Ring of kStages stages; tile lt goes to stage lt % kStages and to consumer warp lt % 4.
+// kStages is a multiple of the number of consumer warps, so each stage (and its pair of
+// barriers) belongs to exactly one warp, which waits on its phases strictly in order: a
+// warp can never be two phases behind a barrier it polls (parity would alias).
+template <int D> struct DecodeCfg {
+    static constexpr int kStagesPerWarp = (D == 128) ? 1 : 2;
+    static constexpr int kStages = kConsumers * kStagesPerWarp;
+    static constexpr int kBoxes = D / 64;                     // 64-element (128 B) boxes per row
+    static constexpr int kTileBytes = TK * D * 2;             // one K (or V) tile
+    static constexpr int kStageBytes = 2 * kTileBytes;
+    static constexpr int kRingBytes = kStages * kStageBytes;
+    static constexpr int kSmemBytes = kRingBytes + 1024 /*align*/ + 2 * kStages * 8;
+    static_assert(kStages % kConsumers == 0, "stages must be owned by single warps");
+    static_assert(kRingBytes >= kConsumers * 16 * D * 4 + 2 * kConsumers * 16 * 4,
+                  "reduction buffer must fit in the ring");
+};
+
+// Byte offset of 16-byte chunk `c` (of D/8) in key row `j` of a tile written by TMA with
+// 128-byte swizzle: boxes of 64 elements, each TK rows of 128 B; chunk index XOR (row % 8).
+__device__ __forceinline__ uint32_t swz(int j, int c) {
+    return (uint32_t)((c >> 3) * (TK * 128) + j * 128 + (((c & 7) ^ (j & 7)) << 4));
+}
+
+template <typename T, int D>
+__global__ void __launch_bounds__(kThreads)
+fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                  const T *__restrict__ q, T *__restrict__ o, float *__restrict__ lse,
+                  float *__restrict__ part_o, float *__restrict__ part_lse, int Hq, int Hkv,
+                  int Nq, int Nkv, int n_tiles, int tiles_per_split, int splits,
+                  float scale_log2, int causal, int *status) {
+    using Cfg = DecodeCfg<D>;
+    constexpr int S = Cfg::kStages;
+    extern __shared__ uint8_t smem_raw[];
+    // 1024-byte alignment of the ring in the shared window (the 128-byte swizzle atom)
+    const uint32_t raw_u32 = fav::smem_u32(smem_raw);
+    uint8_t *ring = smem_raw + ((1024u - (raw_u32 & 1023u)) & 1023u);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(ring + Cfg::kRingBytes);
+    const uint32_t ring_u32 = fav::smem_u32(ring);
+    const uint32_t full0 = fav::smem_u32(bars), empty0 = full0 + 8 * S;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int split = blockIdx.x;
+    const int bkv = blockIdx.y;                  // b * Hkv + g
+    const int b = bkv / Hkv, g = bkv % Hkv;
+    const int G = Hq / Hkv;
+    const int M = Nq * G;                        // query rows that read this KV head
+    const int m0 = blockIdx.z * 16;
+    const int tile0 = split * tiles_per_split;
+    const int my_tiles = min(tiles_per_split, n_tiles - tile0);
+
+    if (threadIdx.x == 0) {
+        (void)FAV_CHECK((ring_u32 & 1023u) == 0, status);
+        (void)FAV_CHECK((ring_u32 - raw_u32) + Cfg::kRingBytes + 16 * S <= fav::dynamic_smem_bytes(), status);
+        for (int s = 0; s < S; ++s) {
+            fav::mbar_init(full0 + 8 * s, 1);
+            fav::mbar_init(empty0 + 8 * s, 1);
+        }
+        fav::mbar_fence_init();
+    }
+    __syncthreads();
+
+    if (warp == kConsumers) {
+        // ---------------- producer: one lane streams K/V tiles with TMA ----------------
+        if (lane == 0) {
+            fav::tma_prefetch_desc(&tmK);
+            fav::tma_prefetch_desc(&tmV);
+            for (int lt = 0; lt < my_tiles; ++lt) {
+                const int st = lt % S;
+                if (lt >= S && !fav::mbar_wait(empty0 + 8 * st, ((lt / S) - 1) & 1, status)) break;
+                const uint32_t full = full0 + 8 * st;
+                fav::mbar_arrive_expect_tx(full, Cfg::kStageBytes);
+                const int key0 = (tile0 + lt) * TK;
+                const uint32_t kdst = ring_u32 + st * Cfg::kStageBytes;
+                const uint32_t vdst = kdst + Cfg::kTileBytes;
+#pragma unroll
+                for (int bx = 0; bx < Cfg::kBoxes; ++bx) {
+                    if (!FAV_CHECK(vdst + (bx + 1) * TK * 128 <= ring_u32 + Cfg::kRingBytes &&
+                                       ((kdst | vdst) & 1023u) == 0 && key0 < n_tiles * TK &&
+                                       bkv < (int)gridDim.y, status))
+                        continue;
+                    fav::tma_load_3d(kdst + bx * TK * 128, &tmK, full, bx * 64, key0, bkv);
+                    fav::tma_load_3d(vdst + bx * TK * 128, &tmV, full, bx * 64, key0, bkv);
+                }
+            }
+        }
+        return;
+    }
+
+    // ---------------- consumers ----------------
+    const int r = lane >> 2, t = lane & 3;
+    // The two MMA rows this thread holds: r and r + 8 of the block's 16-row chunk.
+    int lim[2];        // keys visible to the row: [0, lim)
+    const T *qrow[2];
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+        const int m = m0 + r + 8 * h2;
+        if (m < M) {
+            const int i = m / G, hh = m % G;
+            qrow[h2] = q + ((long long)(b * Hq + g * G + hh) * Nq + i) * D;
+            lim[h2] = causal ? (Nkv - Nq + i + 1) : Nkv;
+        } else {
+            qrow[h2] = nullptr;
+            lim[h2] = Nkv;
+        }
+    }
+    int lim_min = min(lim[0], lim[1]);
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) lim_min = min(lim_min, __shfl_xor_sync(~0u, lim_min, off));
+
+    uint32_t qa[D / 16][4];
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+        const int c = 16 * kk + 2 * t;
+        const uint32_t *q0 = reinterpret_cast<const uint32_t *>(qrow[0]);
+        const uint32_t *q1 = reinterpret_cast<const uint32_t *>(qrow[1]);
+        qa[kk][0] = q0 ? __ldg(q0 + c / 2) : 0u;
+        qa[kk][1] = q1 ? __ldg(q1 + c / 2) : 0u;
+        qa[kk][2] = q0 ? __ldg(q0 + c / 2 + 4) : 0u;
+        qa[kk][3] = q1 ? __ldg(q1 + c / 2 + 4) : 0u;
+    }
+
+    float acc[D / 8][4];
+#pragma unroll
+    for (int nd = 0; nd < D / 8; ++nd) acc[nd][0] = acc[nd][1] = acc[nd][2] = acc[nd][3] = 0.f;
+    float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+    bool ok = true;
+
+    for (int lt = warp; lt < my_tiles; lt += kConsumers) {
+        const int st = lt % S;
+        if (!fav::mbar_wait(full0 + 8 * st, (lt / S) & 1, status)) { ok = false; break; }
+        const uint32_t kbase = ring_u32 + st * Cfg::kStageBytes;
+        const uint32_t vbase = kbase + Cfg::kTileBytes;
+        const int key0 = (tile0 + lt) * TK;
+
+        // S = Q K^T over the tile: 8 n-tiles of 8 keys, fp32 accumulate.
+        float s[TK / 8][4];
+#pragma unroll
+        for (int nt = 0; nt < TK / 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+#pragma unroll
+        for (int kp = 0; kp < D / 32; ++kp) {
+#pragma unroll
+            for (int nt = 0; nt < TK / 8; ++nt) {
+                uint32_t bfr[4] = {0u, 0u, 0u, 0u};
+                const uint32_t la = kbase + swz(8 * nt + (lane & 7), 4 * kp + (lane >> 3));
+                if (FAV_CHECK(la >= ring_u32 && la + 16 <= vbase && (la & 15u) == 0, status))
+                    fav::ldmatrix_x4(bfr, la);
+                fav::mma16816<T>(s[nt], qa[2 * kp], bfr[0], bfr[1]);
+                fav::mma16816<T>(s[nt], qa[2 * kp + 1], bfr[2], bfr[3]);
+            }
+        }
+
+        // Mask, scale into the log2 domain, online softmax.
+        const bool need_mask = key0 + TK > lim_min;
+        float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+        for (int nt = 0; nt < TK / 8; ++nt) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                float x = s[nt][e] * scale_log2;
+                if (need_mask) {
+                    const int j = key0 + 8 * nt + 2 * t + (e & 1);
+                    if (j >= lim[e >> 1]) x = -INFINITY;
+                }
+                s[nt][e] = x;
+                mx[e >> 1] = fmaxf(mx[e >> 1], x);
+            }
+        }
+        float alpha[2], mu[2];
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+            mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(~0u, mx[h2], 1));
+            mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(~0u, mx[h2], 2));
+            const float mn = fmaxf(mrow[h2], mx[h2]);
+            mu[h2] = (mn == -INFINITY) ? 0.f : mn;
+            alpha[h2] = fav::fast_exp2(mrow[h2] - mu[h2]);
+            mrow[h2] = mn;
+            lrow[h2] *= alpha[h2];
+        }
+#pragma unroll
+        for (int nt = 0; nt < TK / 8; ++nt) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float p = fav::fast_exp2(s[nt][e] - mu[e >> 1]);
+                s[nt][e] = p;
+                lrow[e >> 1] += p;
+            }
+        }
+#pragma unroll
+        for (int nd = 0; nd < D / 8; ++nd) {
+            acc[nd][0] *= alpha[0]; acc[nd][1] *= alpha[0];
+            acc[nd][2] *= alpha[1]; acc[nd][3] *= alpha[1];
+        }
+
+        // O += P V: P (rounded to T) is the A operand straight from the S accumulators.
+#pragma unroll
+        for (int ks = 0; ks < TK / 16; ++ks) {
+            uint32_t pa[4];
+            pa[0] = fav::Elem<T>::pack(s[2 * ks][0], s[2 * ks][1]);
+            pa[1] = fav::Elem<T>::pack(s[2 * ks][2], s[2 * ks][3]);
+            pa[2] = fav::Elem<T>::pack(s[2 * ks + 1][0], s[2 * ks + 1][1]);
+            pa[3] = fav::Elem<T>::pack(s[2 * ks + 1][2], s[2 * ks + 1][3]);
+            const int i4 = lane >> 3;
+            const int krow = 16 * ks + ((i4 & 1) << 3) + (lane & 7);
+#pragma unroll
+            for (int np = 0; np < D / 16; ++np) {
+                uint32_t bfr[4] = {0u, 0u, 0u, 0u};
+                const uint32_t la = vbase + swz(krow, 2 * np + (i4 >> 1));
+                if (FAV_CHECK(la >= vbase && la + 16 <= ring_u32 + Cfg::kRingBytes && (la & 15u) == 0, status))
+                    fav::ldmatrix_x4_trans(bfr, la);
+                fav::mma16816<T>(acc[2 * np], pa, bfr[0], bfr[1]);
+                fav::mma16816<T>(acc[2 * np + 1], pa, bfr[2], bfr[3]);
+            }
+        }
+        __syncwarp();
+        if (lane == 0) fav::mbar_arrive(empty0 + 8 * st);
+    }
+
+    // ---------------- merge the four warp states through shared memory ----------------
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+        lrow[h2] += __shfl_xor_sync(~0u, lrow[h2], 1);
+        lrow[h2] += __shfl_xor_sync(~0u, lrow[h2], 2);
+    }
+    fav::named_bar_sync(1, kConsumers * 32);   // every consumer is done with the ring
+    float *red = reinterpret_cast<float *>(ring);          // [warp][16][D]
+    float *redm = red + kConsumers * 16 * D;                // [warp][16]
+    float *redl = redm + kConsumers * 16;                   // [warp][16]
+    float *mine = red + warp * 16 * D;
+#pragma unroll
+    for (int nd = 0; nd < D / 8; ++nd) {
+        const int c = 8 * nd + 2 * t;
+        *reinterpret_cast<float2 *>(mine + r * D + c) = make_float2(acc[nd][0], acc[nd][1]);
+        *reinterpret_cast<float2 *>(mine + (r + 8) * D + c) = make_float2(acc[nd][2], acc[nd][3]);
+    }
+    if (t == 0) {
+        redm[warp * 16 + r] = mrow[0];
+        redm[warp * 16 + r + 8] = mrow[1];
+        redl[warp * 16 + r] = lrow[0];
+        redl[warp * 16 + r + 8] = lrow[1];
+    }
+    fav::named_bar_sync(1, kConsumers * 32);
+    if (!ok) return;
+
+    constexpr int kCols = D / 8;                 // columns per thread (8 threads per row)
+    const int rr = threadIdx.x >> 3;             // 0..15
+    const int c0 = (threadIdx.x & 7) * kCols;
+    const int m = m0 + rr;
+    if (m >= M) return;
+    float mw[kConsumers], Mx = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kConsumers; ++w) {
+        mw[w] = redm[w * 16 + rr];
+        Mx = fmaxf(Mx, mw[w]);
+    }
+    float ew[kConsumers], L = 0.f;
+#pragma unroll
+    for (int w = 0; w < kConsumers; ++w) {
+        ew[w] = (Mx == -INFINITY) ? 0.f : exp2f(mw[w] - Mx);
+        L += ew[w] * redl[w * 16 + rr];
+    }
+    const float invL = (L > 0.f) ? 1.f / L : 0.f;
+    float out[kCols];
+#pragma unroll
+    for (int c = 0; c < kCols; ++c) {
+        float x = 0.f;
+#pragma unroll
+        for (int w = 0; w < kConsumers; ++w) x += ew[w] * red[(w * 16 + rr) * D + c0 + c];
+        out[c] = x * invL;
+    }
+    const int i = m / G, hh = m % G;
+    const long long flat = (long long)(b * Hq + g * G + hh) * Nq + i;
+    const long long rows_total = (long long)gridDim.y * G * Nq;
+    (void)rows_total;
+    if (!FAV_CHECK(flat >= 0 && flat < rows_total && c0 + kCols <= D, status)) return;
+    const float lse_val = (L > 0.f) ? (Mx + log2f(L)) * kLn2 : -INFINITY;
+    if (splits == 1) {
+        T *orow = o + flat * D + c0;
+#pragma unroll
+        for (int c = 0; c < kCols; c += 8) {
+            uint4 pk;
+            pk.x = fav::Elem<T>::pack(out[c + 0], out[c + 1]);
+            pk.y = fav::Elem<T>::pack(out[c + 2], out[c + 3]);
+            pk.z = fav::Elem<T>::pack(out[c + 4], out[c + 5]);
+            pk.w = fav::Elem<T>::pack(out[c + 6], out[c + 7]);
+            *reinterpret_cast<uint4 *>(orow + c) = pk;
+        }
+        if (lse && (threadIdx.x & 7) == 0) lse[flat] = lse_val;
+    } else {
+        float *prow = part_o + (flat * splits + split) * D + c0;
+#pragma unroll
+        for (int c = 0; c < kCols; c += 4)
+            *reinterpret_cast<float4 *>(prow + c) = make_float4(out[c], out[c + 1], out[c + 2], out[c + 3]);
+        if ((threadIdx.x & 7) == 0) part_lse[flat * splits + split] = lse_val;
+    }
+}
+
+// One warp per query row: L = logsumexp over splits, O = sum_s exp(lse_s - L) O_s.
+template <typename T, int D>
+__global__ void __launch_bounds__(128)
+fav_combine_kernel(const float *__restrict__ part_o, const float *__restrict__ part_lse,
+                   T *__restrict__ o, float *__restrict__ lse, long long rows, int splits) {
+    const long long row = (long long)blockIdx.x * 4 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= rows) return;
+    const float *pl = part_lse + row * splits;
+    float mx = -INFINITY;
+    for (int s = lane; s < splits; s += 32) mx = fmaxf(mx, pl[s]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(~0u, mx, off));
+    float sum = 0.f;
+    for (int s = lane; s < splits; s += 32) sum += (pl[s] == -INFINITY) ? 0.f : expf(pl[s] - mx);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(~0u, sum, off);
+    const float L = mx + logf(sum);
+    constexpr int kPer = D / 32;                  // consecutive columns per lane
+    float accv[kPer];
+#pragma unroll
+    for (int c = 0; c < kPer; ++c) accv[c] = 0.f;
+    const float *po = part_o + row * splits * D + lane * kPer;
+    for (int s0 = 0; s0 < splits; s0 += 32) {
+        const int s = s0 + lane;
+        const float wl = (s < splits && pl[s] != -INFINITY) ? expf(pl[s] - L) : 0.f;
+        const int cnt = min(32, splits - s0);
+        for (int jj = 0; jj < cnt; ++jj) {
+            const float w = __shfl_sync(~0u, wl, jj);
+            const float *src = po + (long long)(s0 + jj) * D;
+#pragma unroll
+            for (int c = 0; c < kPer; c += 2) {
+                const float2 x = *reinterpret_cast<const float2 *>(src + c);
+                accv[c] = fmaf(w, x.x, accv[c]);
+                accv[c + 1] = fmaf(w, x.y, accv[c + 1]);
+            }
+        }
+    }
+    T *orow = o + row * D + lane * kPer;
+#pragma unroll
+    for (int c = 0; c < kPer; c += 2)
+        *reinterpret_cast<uint32_t *>(orow + c) = fav::Elem<T>::pack(accv[c], accv[c + 1]);
+    if (lse && lane == 0) lse[row] = L;
+}
+
+template <typename T, int D>
+fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t stream) {
+    using Cfg = DecodeCfg<D>;
+    alignas(64) CUtensorMap tmK, tmV;
+    const int outer = a.B * a.Hkv;
+    fav_status st = fav_make_tmap_3d(&tmK, a.k, D, a.Nkv, outer, TK);
+    if (st != FAV_OK) return st;
+    st = fav_make_tmap_3d(&tmV, a.v, D, a.Nkv, outer, TK);
+    if (st != FAV_OK) return st;
+    const int n_tiles = fav_decode_num_tiles(a);
+    const int tps = (n_tiles + splits - 1) / splits;
+    splits = (n_tiles + tps - 1) / tps;
+    const int M = a.Nq * (a.Hq / a.Hkv);
+    const int chunks = (M + 15) / 16;
+    auto kern = fav_decode_kernel<T, D>;
+    static bool attr_set = false;   // per-process; the attribute is per function, not per device
+    if (!attr_set) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 Cfg::kSmemBytes) != cudaSuccess)
+            return FAV_ERR_CUDA;
+        attr_set = true;
+    }
+    const long long rows = (long long)a.B * a.Hq * a.Nq;
+    float *part_o = reinterpret_cast<float *>(workspace);
+    float *part_lse = part_o ? part_o + rows * splits * D : nullptr;
+    const float scale_log2 = a.scale * kLog2e;
+    dim3 grid(splits, outer, chunks);
+    kern<<<grid, kThreads, Cfg::kSmemBytes, stream>>>(
+        tmK, tmV, (const T *)a.q, (T *)a.o, a.lse, part_o, part_lse, a.Hq, a.Hkv, a.Nq, a.Nkv,
+        n_tiles, tps, splits, scale_log2, a.causal, a.dev_status);
+    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_decode_kernel", stream))
+        return FAV_ERR_CUDA;
+    if (splits > 1) {
+        const unsigned blocks = (unsigned)((rows + 3) / 4);
+        fav_combine_kernel<T, D><<<blocks, 128, 0, stream>>>(part_o, part_lse, (T *)a.o, a.lse,
+                                                              rows, splits);
+        if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_combine_kernel", stream))
+            return FAV_ERR_CUDA;
+    }
+    return FAV_OK;
+}
+
+}  // namespace
+
+bool fav_decode_supported(const FavArgs &a) {
+    if (a.dtype != FAV_F16 && a.dtype != FAV_BF16) return false;
+    if (a.D != 64 && a.D != 128) return false;
+    const long long M = (long long)a.Nq * (a.Hq / a.Hkv);
+    return M <= 64 && (long long)a.B * a.Hkv <= 65535;
+}
+
+int fav_decode_num_tiles(const FavArgs &a) { return (a.Nkv + TK - 1) / TK; }
+
+// Enough blocks for several waves of two resident blocks per SM, at least two tiles each.
+int fav_decode_auto_splits(const FavArgs &a) {
+    const int n_tiles = fav_decode_num_tiles(a);
+    const long long M = (long long)a.Nq * (a.Hq / a.Hkv);
+    const long long groups = (long long)a.B * a.Hkv * ((M + 15) / 16);
+    const long long target = 8LL * (a.num_sms > 0 ? a.num_sms : 148);
+    long long splits = (target + groups - 1) / groups;
+    splits = std::min<long long>(splits, std::max(1, n_tiles / 2));
+    splits = std::max<long long>(1, std::min<long long>(splits, 4096));
+    return (int)splits;
+}
+
+size_t fav_decode_workspace_bytes(const FavArgs &a, int splits) {
+    if (splits <= 1) return 0;
+    const size_t rows = (size_t)a.B * a.Hq * a.Nq;
+    return rows * splits * ((size_t)a.D + 1) * sizeof(float);
+}
+
+fav_status fav_launch_decode(const FavArgs &a, int splits, void *workspace, cudaStream_t s) {
+    if (a.dtype == FAV_F16)
+        return a.D == 128 ? launch<__half, 128>(a, splits, workspace, s)
+                          : launch<__half, 64>(a, splits, workspace, s);
+    return a.D == 128 ? launch<__nv_bfloat16, 128>(a, splits, workspace, s)
+                      : launch<__nv_bfloat16, 64>(a, splits, workspace, s);
+}

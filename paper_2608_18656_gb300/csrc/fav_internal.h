@@ -1,0 +1,43 @@
+// fav_internal.h -- host-side interface between the C ABI (fav_api.cu) and the kernel files.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/fav.h"
+
+struct FavArgs {
+    const void *q, *k, *v;
+    void *o;
+    float *lse;
+    int B, Hq, Hkv, Nq, Nkv, D;
+    float scale;
+    int causal;
+    fav_dtype dtype;
+    int *dev_status;   // device word set by bounded waits that gave up
+    int num_sms;
+};
+
+// Generic CUDA-core kernel (fav_simt.cu).
+bool fav_simt_supported(const FavArgs &a);
+fav_status fav_launch_simt(const FavArgs &a, cudaStream_t s);
+
+// Split-KV decode kernel + combine (fav_decode.cu).
+bool fav_decode_supported(const FavArgs &a);
+int fav_decode_num_tiles(const FavArgs &a);
+int fav_decode_auto_splits(const FavArgs &a);
+size_t fav_decode_workspace_bytes(const FavArgs &a, int splits);
+fav_status fav_launch_decode(const FavArgs &a, int splits, void *workspace, cudaStream_t s);
+
+// tcgen05 prefill kernel (fav_prefill.cu).
+bool fav_prefill_supported(const FavArgs &a);
+fav_status fav_launch_prefill(const FavArgs &a, cudaStream_t s);
+
+// With FAV_DEBUG_SYNC=1 in the environment: synchronise `s` after a launch and report a
+// failure of kernel `what` on stderr.  Returns true if the kernel failed.  No-op otherwise.
+bool fav_debug_sync(const char *what, cudaStream_t s);
+
+// Tensor-map encoding through the driver entry point (fav_api.cu).
+// 3-D map over a [outer, rows, D] tensor of 16-bit elements, box {64, box_rows, 1},
+// 128-byte swizzle, zero fill out of bounds.
+fav_status fav_make_tmap_3d(void *tmap /* CUtensorMap* */, const void *base, int D, int rows,
+                            int outer, int box_rows);

@@ -1,0 +1,146 @@
+"""Parity of the CUDA path with the fp64 oracle on seeded inputs (needs a GB300)."""
+import numpy as np
+import pytest
+
+import paper_2608_18656_gb300 as fav
+from paper_2608_18656_gb300 import inputs as I
+from gpu_util import check, run_gpu, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _reset():
+    fav.set_path(fav.PATH_AUTO)
+    fav.set_decode_splits(0)
+    yield
+    fav.set_path(fav.PATH_AUTO)
+    fav.set_decode_splits(0)
+
+
+def W(dtype, B, Hq, Hkv, Nq, Nkv, D, causal=False, outliers=False, seed=7):
+    return I.Workload("t", dtype, B, Hq, Hkv, Nq, Nkv, D, causal, outliers, seed)
+
+
+# ---- the five measured workloads at full size ----
+
+def test_workload0_fp32_mha_full():
+    w = I.WORKLOADS[0]
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_SIMT
+    check(w, o, lse, x)
+
+
+@pytest.mark.parametrize("idx", [1, 2])
+def test_prefill_workloads_full_sampled(idx):
+    w = I.WORKLOADS[idx]
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    check(w, o, lse, x, rows=sample_rows(w, 4096, seed=idx))
+
+
+@pytest.mark.parametrize("idx", [3, 4])
+def test_decode_workloads_full(idx):
+    w = I.WORKLOADS[idx]
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_DECODE
+    assert fav.last_decode_splits() > 1
+    check(w, o, lse, x)
+
+
+# ---- decode path edge cases ----
+
+@pytest.mark.parametrize("dtype", [I.F16, I.BF16])
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("G", [1, 2, 4, 8, 16])
+def test_decode_group_sizes(dtype, D, G):
+    w = W(dtype, 2, 2 * G, 2, 1, 1000, D, seed=G + D)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_DECODE
+    check(w, o, lse, x)
+
+
+@pytest.mark.parametrize("splits", [1, 2, 3, 7, 16, 1000])
+def test_decode_split_counts(splits):
+    fav.set_decode_splits(splits)
+    w = W(I.BF16, 1, 8, 1, 1, 777, 128, seed=splits)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    assert 1 <= fav.last_decode_splits() <= splits
+    check(w, o, lse, x)
+
+
+@pytest.mark.parametrize("Nkv", [1, 2, 31, 32, 33, 63, 64, 65, 129])
+def test_decode_short_caches(Nkv):
+    w = W(I.F16, 1, 4, 1, 1, Nkv, 128, seed=Nkv)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    check(w, o, lse, x)
+
+
+@pytest.mark.parametrize("Nq,G,causal", [(2, 4, True), (4, 4, True), (3, 1, False),
+                                         (4, 8, True), (16, 4, True)])
+def test_decode_path_small_nq(Nq, G, causal):
+    """Several queries per KV head (speculative-decode shape), bottom-right causal."""
+    fav.set_path(fav.PATH_DECODE)
+    w = W(I.BF16, 2, 2 * G, 2, Nq, 300, 64, causal=causal, seed=Nq * 10 + G)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_DECODE
+    check(w, o, lse, x)
+
+
+def test_decode_without_lse():
+    w = W(I.F16, 1, 8, 2, 1, 500, 128, seed=3)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x, return_lse=False)
+    assert lse is None
+    check(w, o, None, x)
+
+
+def test_decode_outliers():
+    w = W(I.BF16, 2, 16, 1, 1, 4096, 128, outliers=True, seed=5)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    check(w, o, lse, x)
+
+
+# ---- CUDA-core path ----
+
+@pytest.mark.parametrize("dtype", [I.F32, I.F16, I.BF16])
+@pytest.mark.parametrize("shape", [(1, 2, 2, 1, 1, 64, False), (2, 4, 2, 37, 37, 32, True),
+                                   (1, 3, 1, 5, 200, 8, True), (1, 2, 2, 128, 128, 256, False),
+                                   (1, 1, 1, 33, 70, 96, False)])
+def test_simt_path(dtype, shape):
+    fav.set_path(fav.PATH_SIMT)
+    B, Hq, Hkv, Nq, Nkv, D, causal = shape
+    if dtype != I.F32 and D % 8:
+        pytest.skip("16-bit rows need D % 8 == 0")
+    w = W(dtype, B, Hq, Hkv, Nq, Nkv, D, causal=causal, seed=Nq + D)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_SIMT
+    check(w, o, lse, x)
+
+
+def test_forced_path_that_cannot_run_is_unsupported():
+    import torch
+    fav.set_path(fav.PATH_DECODE)
+    q = torch.zeros(1, 1, 4, 64, device="cuda", dtype=torch.float32)
+    with pytest.raises(fav.FavError) as e:
+        fav.forward(q, q, q)
+    assert e.value.status == 2
+
+
+def test_error_leaves_outputs_untouched():
+    import torch
+    q = torch.randn(1, 3, 4, 64, device="cuda", dtype=torch.float16)
+    k = torch.randn(1, 2, 4, 64, device="cuda", dtype=torch.float16)
+    o = torch.full_like(q, 7.0)
+    with pytest.raises(fav.FavError):
+        fav.forward(q, k, k, out=o)
+    torch.cuda.synchronize()
+    assert bool((o == 7.0).all())
