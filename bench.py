@@ -244,7 +244,7 @@ def reference_arm(args, dist):
         return
     w = I.WORKLOADS[HEADLINE]
     x = I.make_inputs(w)
-    rows, flops = oracle_sample(w, 2048)
+    rows, flops = oracle_sample(w, w.B * w.Hq * w.Nq)
     for _ in range(args.warmup):
         run_oracle(w, x, rows)
     times = []
@@ -332,10 +332,10 @@ def fav_arm(args, dist):
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
     cpu = None
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu:
-        rows, flops = oracle_sample(w, 2048)
+        rows, flops = oracle_sample(w, w.B * w.Hq * w.Nq)
         t, cores = run_oracle(w, x, rows)
         cpu = {"value": flops / t / 1e12, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
-               "sample": "%d of %d query rows (seeded) of %s, fp64, %.2f s"
+               "sample": "%d of %d query rows of %s, fp64, %.2f s"
                          % (len(rows), w.B * w.Hq * w.Nq, w.name, t)}
     traffic = None
     tpath = os.path.join(ROOT, "profiles", "traffic.json")

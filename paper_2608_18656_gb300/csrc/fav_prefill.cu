@@ -47,16 +47,28 @@ template <int D> struct PrefillCfg {
     static constexpr int kOffK = kOffQ + kQBytes;
     static constexpr int kOffV = kOffK + kStages * kKVBytes;
     static constexpr int kOffP = kOffV + kStages * kKVBytes;
-    static constexpr int kOffBar = kOffP + kPBytes;
+    static constexpr int kOnesBytes = 16 * 128;              // 16 rows x 64 ones (bf16)
+    static constexpr int kOffOnes = kOffP + kPBytes;
+    static constexpr int kOffBar = kOffOnes + 1024 * ((kOnesBytes + 1023) / 1024);
     static constexpr int kNumBars = 1 + 4 * kStages + 2 + 2 + 2;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
     static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
     static constexpr uint32_t kTmemCols = 512;               // S0 | S1 | O
     static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
+    static constexpr uint32_t kColL = kColO + D;             // 16 columns of sum_k P~[row][k]
 };
 
 template <typename T> struct IsBF16 { static constexpr bool value = false; };
 template <> struct IsBF16<__nv_bfloat16> { static constexpr bool value = true; };
+
+// With bf16 I/O the weights P are rounded to 8 significant bits before the P.V product.  With
+// the lazy maximum a dominant weight can be any value up to 2^8, so normalising the rounded
+// numerator by the unrounded fp32 sum would leave the dominant term off by up to 2^-9 of |v|.
+// The bf16 kernel therefore divides by l~ = sum_k P~[row][k], accumulated by the tensor core
+// (P~ times a column of ones) next to O, so numerator and denominator use the same weights;
+// the fp32 sum of the unrounded weights still gives the LSE.  fp16 keeps 11 bits and divides
+// by the fp32 sum.
+template <typename T> struct RoundedNorm { static constexpr bool value = IsBF16<T>::value; };
 
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -114,6 +126,12 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         fav::mbar_init(p_empty, 1);
         fav::mbar_fence_init();
     }
+    if (RoundedNorm<T>::value && warp >= 2) {
+        // bf16 1.0 = 0x3F80; every element of the tile is one, so its layout is irrelevant.
+        uint32_t *ones = reinterpret_cast<uint32_t *>(smem + C::kOffOnes);
+        for (int i = threadIdx.x - 64; i < C::kOnesBytes / 4; i += kThreads - 64) ones[i] = 0x3F803F80u;
+        fav::tc::fence_proxy_async_smem();
+    }
     if (warp == 1) {
         fav::tc::tmem_alloc(fav::smem_u32(tmem_slot), C::kTmemCols);
         fav::tc::tmem_relinquish();
@@ -157,6 +175,8 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             constexpr bool bf = IsBF16<T>::value;
             constexpr uint32_t idesc_qk = fav::tc::idesc_f16(BM, BN, bf, false);
             constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, bf, true);
+            constexpr uint32_t idesc_l = fav::tc::idesc_f16(BM, 16, bf, false);
+            const uint64_t ones_desc = fav::tc::sdesc_sw128(sbase + C::kOffOnes, 16, 1024);
             bool ok = fav::mbar_wait(q_full, 0, status);
             // S_j = Q K_j^T into S buffer j % 2
             auto issue_s = [&](int j) -> bool {
@@ -195,6 +215,8 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                         sP + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
                     const uint64_t bd = fav::tc::sdesc_sw128(vst + kk * 16 * 128, BN * 128, 1024);
                     fav::tc::mma_ss(tmem + C::kColO, ad, bd, idesc_pv, (j > 0 || kk > 0));
+                    if (RoundedNorm<T>::value)
+                        fav::tc::mma_ss(tmem + C::kColL, ad, ones_desc, idesc_l, (j > 0 || kk > 0));
                 }
                 fav::tc::commit(v_empty + 8 * st);
                 fav::tc::commit(p_empty);
@@ -262,8 +284,9 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             if (j > 0 && !fav::mbar_wait(p_empty, (j - 1) & 1, status)) { ok = false; break; }
             fav::tc::fence_after();
             if (__any_sync(~0u, rescale)) {
+                constexpr int kChunks = D / 32 + (RoundedNorm<T>::value ? 1 : 0);   // O (+ l~)
 #pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
+                for (int c = 0; c < kChunks; ++c) {
                     uint32_t r[32];
                     fav::tc::ld_32x32b_x32(trow + C::kColO + c * 32, r);
                     fav::tc::wait_ld();
@@ -291,7 +314,13 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         // ---------------- epilogue: O / l, LSE ----------------
         if (ok && n_kv > 0 && fav::mbar_wait(p_empty, (n_kv - 1) & 1, status)) {
             fav::tc::fence_after();
-            const float inv_l = 1.f / l;
+            float inv_l = 1.f / l;
+            if (RoundedNorm<T>::value) {
+                uint32_t r[32];
+                fav::tc::ld_32x32b_x32(trow + C::kColL, r);
+                fav::tc::wait_ld();
+                inv_l = 1.f / __uint_as_float(r[0]);
+            }
             const bool valid = qi < Nq;
             T *orow = o + ((long long)bh * Nq + qi) * D;
 #pragma unroll
