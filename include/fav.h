@@ -126,6 +126,31 @@ FAV_API fav_status fav_set_decode_splits(int n);
 /* The split count the last decode-path fav_forward call used (0 if none ran yet). */
 FAV_API int fav_last_decode_splits(void);
 
+/*
+ * fav_decode_noalloc -- the decode path (split-KV decode kernel + log-sum-exp combine) with no
+ * device allocation at all.  The paper has no counterpart: this entry point exists for callers
+ * that cannot let a library allocate device memory -- a server whose own pool reserves all
+ * device memory at start-up (a library cudaMalloc would fail or compete with it), or a
+ * latency-critical decode loop that forbids allocator calls after initialisation.
+ *
+ * Same arguments, layouts, ownership and status codes as fav_forward, for decode-shaped calls
+ * (fp16/bf16, D in {64, 128}, Nq * Hq / Hkv <= 64); the result equals fav_forward's on the
+ * decode path.  The split-KV partials live in a fixed file-scope device array of
+ * FAV_NOALLOC_SCRATCH_BYTES (16 MiB), held by every GPU that loads the library until the
+ * process exits.  The split count is fav_forward's (automatic, or fav_set_decode_splits);
+ * FAV_ERR_UNSUPPORTED if its partials, B*Hq*Nq * splits * (D + 1) * 4 bytes, exceed the array,
+ * or if the call is not decode-shaped.  The first call on each device (with that device
+ * current) looks up the array's device address; make that first call before any stream
+ * capture.  Every call shares the array: calls that overlap on the GPU (several streams at
+ * once) race and must be serialised by the caller.  Never calls cudaMalloc, cudaMallocAsync,
+ * cudaFree or any allocating library routine.
+ */
+#define FAV_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+FAV_API fav_status fav_decode_noalloc(const void *q, const void *k, const void *v, void *o,
+                                      float *lse, int B, int Hq, int Hkv, int Nq, int Nkv,
+                                      int D, float scale, int causal, fav_dtype dtype,
+                                      void *stream);
+
 #ifdef __cplusplus
 }
 #endif

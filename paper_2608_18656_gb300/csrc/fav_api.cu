@@ -168,6 +168,22 @@ fav_status forward_impl(const FavArgs &in, cudaStream_t stream) {
 
 }  // namespace
 
+fav_status fav_internal_validate(int B, int Hq, int Hkv, int Nq, int Nkv, int D, float scale,
+                                 int causal, fav_dtype dtype) {
+    return validate_shape(B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+}
+
+fav_status fav_internal_device_info(int **dev_status, int *num_sms) {
+    DeviceState *ds = nullptr;
+    const fav_status st = device_state(&ds);
+    if (st != FAV_OK) return st;
+    *dev_status = ds->status;
+    *num_sms = ds->num_sms;
+    return FAV_OK;
+}
+
+int fav_internal_decode_splits_override() { return g_splits.load(); }
+
 bool fav_debug_sync(const char *what, cudaStream_t s) {
     static const bool on = [] {
         const char *e = getenv("FAV_DEBUG_SYNC");

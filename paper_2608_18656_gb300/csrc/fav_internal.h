@@ -36,6 +36,14 @@ fav_status fav_launch_prefill(const FavArgs &a, cudaStream_t s);
 // failure of kernel `what` on stderr.  Returns true if the kernel failed.  No-op otherwise.
 bool fav_debug_sync(const char *what, cudaStream_t s);
 
+// Shared with the allocation-free decode entry point (fav_noalloc.cu), defined in fav_api.cu:
+// the same shape/argument rules as fav_forward, the device's status word and SM count, and
+// the process-wide decode split override (0 = automatic).
+fav_status fav_internal_validate(int B, int Hq, int Hkv, int Nq, int Nkv, int D, float scale,
+                                 int causal, fav_dtype dtype);
+fav_status fav_internal_device_info(int **dev_status, int *num_sms);
+int fav_internal_decode_splits_override();
+
 // Tensor-map encoding through the driver entry point (fav_api.cu).
 // 3-D map over a [outer, rows, D] tensor of 16-bit elements, box {64, box_rows, 1},
 // 128-byte swizzle, zero fill out of bounds.
