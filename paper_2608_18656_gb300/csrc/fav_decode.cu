@@ -82,6 +82,9 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     const int tile0 = split * tiles_per_split;
     const int my_tiles = min(tiles_per_split, n_tiles - tile0);
 
+    // Let a dependent combine grid be scheduled once every block of this grid has started; it
+    // still waits for this grid's completion before reading anything.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (threadIdx.x == 0) {
         (void)FAV_CHECK((ring_u32 & 1023u) == 0, status);
         (void)FAV_CHECK((ring_u32 - raw_u32) + Cfg::kRingBytes + 16 * S <= fav::dynamic_smem_bytes(), status);
@@ -328,49 +331,70 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     }
 }
 
-// One warp per query row: L = logsumexp over splits, O = sum_s exp(lse_s - L) O_s.
+// One block per query row: L = logsumexp_s lse_s, O = sum_s exp(lse_s - L) O_s.  The four
+// warps take every fourth split, each lane a group of D/32 consecutive columns (vector
+// loads); the warp sums are added in shared memory.  Launched as a programmatic dependent of
+// the decode kernel: it may be scheduled while the decode grid drains, and waits for that
+// grid's completion (and memory) before reading the partials.
 template <typename T, int D>
 __global__ void __launch_bounds__(128)
 fav_combine_kernel(const float *__restrict__ part_o, const float *__restrict__ part_lse,
                    T *__restrict__ o, float *__restrict__ lse, long long rows, int splits) {
-    const long long row = (long long)blockIdx.x * 4 + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    __shared__ float red[4][D];
+    __shared__ float wred[4];
+    const long long row = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (row >= rows) return;
     const float *pl = part_lse + row * splits;
     float mx = -INFINITY;
-    for (int s = lane; s < splits; s += 32) mx = fmaxf(mx, pl[s]);
+    for (int s = threadIdx.x; s < splits; s += 128) mx = fmaxf(mx, pl[s]);
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(~0u, mx, off));
+    if (lane == 0) wred[warp] = mx;
+    __syncthreads();
+    mx = fmaxf(fmaxf(wred[0], wred[1]), fmaxf(wred[2], wred[3]));
+    __syncthreads();
     float sum = 0.f;
-    for (int s = lane; s < splits; s += 32) sum += (pl[s] == -INFINITY) ? 0.f : expf(pl[s] - mx);
+    for (int s = threadIdx.x; s < splits; s += 128)
+        sum += (pl[s] == -INFINITY) ? 0.f : expf(pl[s] - mx);
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(~0u, sum, off);
-    const float L = mx + logf(sum);
+    if (lane == 0) wred[warp] = sum;
+    __syncthreads();
+    const float L = mx + logf(wred[0] + wred[1] + wred[2] + wred[3]);
     constexpr int kPer = D / 32;                  // consecutive columns per lane
-    float accv[kPer];
+    float acc[kPer];
 #pragma unroll
-    for (int c = 0; c < kPer; ++c) accv[c] = 0.f;
+    for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
     const float *po = part_o + row * splits * D + lane * kPer;
-    for (int s0 = 0; s0 < splits; s0 += 32) {
-        const int s = s0 + lane;
-        const float wl = (s < splits && pl[s] != -INFINITY) ? expf(pl[s] - L) : 0.f;
-        const int cnt = min(32, splits - s0);
-        for (int jj = 0; jj < cnt; ++jj) {
-            const float w = __shfl_sync(~0u, wl, jj);
-            const float *src = po + (long long)(s0 + jj) * D;
-#pragma unroll
-            for (int c = 0; c < kPer; c += 2) {
-                const float2 x = *reinterpret_cast<const float2 *>(src + c);
-                accv[c] = fmaf(w, x.x, accv[c]);
-                accv[c + 1] = fmaf(w, x.y, accv[c + 1]);
-            }
+#pragma unroll 4
+    for (int s = warp; s < splits; s += 4) {
+        const float ls = pl[s];
+        const float w = (ls == -INFINITY) ? 0.f : expf(ls - L);
+        const float *src = po + (long long)s * D;
+        if constexpr (kPer == 4) {
+            const float4 x = *reinterpret_cast<const float4 *>(src);
+            acc[0] = fmaf(w, x.x, acc[0]);
+            acc[1] = fmaf(w, x.y, acc[1]);
+            acc[2] = fmaf(w, x.z, acc[2]);
+            acc[3] = fmaf(w, x.w, acc[3]);
+        } else {
+            const float2 x = *reinterpret_cast<const float2 *>(src);
+            acc[0] = fmaf(w, x.x, acc[0]);
+            acc[1] = fmaf(w, x.y, acc[1]);
         }
     }
-    T *orow = o + row * D + lane * kPer;
 #pragma unroll
-    for (int c = 0; c < kPer; c += 2)
-        *reinterpret_cast<uint32_t *>(orow + c) = fav::Elem<T>::pack(accv[c], accv[c + 1]);
-    if (lse && lane == 0) lse[row] = L;
+    for (int c = 0; c < kPer; ++c) red[warp][lane * kPer + c] = acc[c];
+    __syncthreads();
+    if (threadIdx.x < D / 2) {
+        const int c = threadIdx.x * 2;
+        const float x0 = red[0][c] + red[1][c] + red[2][c] + red[3][c];
+        const float x1 = red[0][c + 1] + red[1][c + 1] + red[2][c + 1] + red[3][c + 1];
+        *reinterpret_cast<uint32_t *>(o + row * D + c) = fav::Elem<T>::pack(x0, x1);
+    }
+    if (lse && threadIdx.x == 0) lse[row] = L;
 }
 
 template <typename T, int D>
@@ -406,9 +430,21 @@ fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t st
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_decode_kernel", stream))
         return FAV_ERR_CUDA;
     if (splits > 1) {
-        const unsigned blocks = (unsigned)((rows + 3) / 4);
-        fav_combine_kernel<T, D><<<blocks, 128, 0, stream>>>(part_o, part_lse, (T *)a.o, a.lse,
-                                                              rows, splits);
+        if (rows > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)rows);
+        cfg.blockDim = dim3(128);
+        cfg.dynamicSmemBytes = 0;
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        T *out = (T *)a.o;
+        float *lse_out = a.lse;
+        cudaLaunchKernelEx(&cfg, fav_combine_kernel<T, D>, (const float *)part_o,
+                           (const float *)part_lse, out, lse_out, rows, splits);
         if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_combine_kernel", stream))
             return FAV_ERR_CUDA;
     }

@@ -5,110 +5,170 @@
 // the scores are computed, the running maximum / sum / output accumulator of the online
 // softmax are updated (rescale by exp(M_old - M), weights exp(S - M)), and after the last
 // block the accumulator is normalised.  Heads sharing a K/V head read the same K/V tiles
-// (GQA reuse).  On this GPU the paper's register blocking becomes:
-//   * a 128 x D query tile in shared memory (TMA, 128-byte swizzle), loaded once;
-//   * 128-key K and V tiles streamed by TMA through a ring of shared-memory stages;
-//   * S = Q K^T (M = 128, N = 128, K = D) and O += P V (M = 128, N = D, K = 128) as
-//     tcgen05.mma issued by one thread, accumulating in tensor memory (TMEM):
-//     two S buffers (so S_{j+1} is computed while the softmax works on S_j) and one O;
-//   * a softmax warpgroup, one thread per query row (= TMEM lane): tcgen05.ld of its S row,
-//     mask, row max, exp2 in the log2 domain, row sum, P rounded to the I/O type and written
-//     to shared memory in the K-major 128-byte-swizzled layout the MMA reads.
+// (GQA reuse), and several heads are processed by one unit of work (the paper's inter-head
+// parallelism).  On this GPU that becomes:
+//   * each CTA owns two 128-row query tiles that read the same K/V head: the same query tile
+//     of two heads of one GQA group (even group sizes), or two consecutive query tiles of one
+//     head (MHA).  Both Q tiles live in shared memory (TMA, 128-byte swizzle), loaded once;
+//   * 128-key K and V tiles are streamed by TMA through a ring of shared-memory stages and
+//     serve both query tiles;
+//   * S_i = Q_i K^T (M = 128, N = 128, K = D) and O_i += P_i V (M = 128, N = D, K = 128) are
+//     tcgen05.mma issued by one thread, accumulating in tensor memory (TMEM).  P_i is written
+//     back into TMEM over the columns of S_i and read from there by the P.V MMA;
+//   * one softmax warpgroup per query tile, one thread per query row (= TMEM lane): tcgen05.ld
+//     of its S row, mask, row max, exp2 in the log2 domain, row sum, P rounded to the I/O type,
+//     tcgen05.st of P.  The MMA thread alternates between the two tiles (P.V and the next
+//     Q.K^T of tile 0 while the softmax works on tile 1, and vice versa), so the tensor core
+//     and the softmax overlap.
 // The running maximum is updated lazily: O and l are rescaled only when the maximum grows by
 // more than 2^8 (log2 domain); otherwise the stale maximum is kept and the weights may reach
 // 256.  The final O / l uses the same maximum as every weight, so the result is unchanged.
+// Because MMAs complete in issue order and S_i(j) is issued after P_i(j-1).V, O_i is stable
+// when S_i(j) arrives: the softmax thread rescales it itself, before writing P_i(j).
 //
-// Warp roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM owner + MMA issuer,
-// warps 2..5 = softmax / correction / epilogue (TMEM lane quarter = warp % 4).
+// Warp roles (320 threads): warps 0-3 softmax of tile 0, warps 4-7 softmax of tile 1
+// (TMEM lane quarter = warp % 4); warp 8 = TMEM owner + MMA issuer (one thread); warp 9 = TMA
+// producer.  The issuing thread blocks while the tensor pipe is busy, and a wait on an
+// mbarrier costs it ~80 cycles of latency even when the phase is already complete; so it
+// tests the barriers it will need next *before* a burst of MMAs and looks at the answers
+// after it, and only waits for real on the ones that were not complete.
 #include <cuda.h>
 #include <math.h>
+
+#include <type_traits>
 
 #include "fav_device.cuh"
 #include "fav_internal.h"
 #include "fav_tc.cuh"
 
+// Timing builds (-DFAV_TIMING) record SM clock stamps at the phase boundaries of the first
+// block's loops and print them at the end; release builds compile this away.
+#ifdef FAV_TIMING
+#define FAV_STAMP(arr, j, k) do { if ((j) < 16) (arr)[j][k] = clock64(); } while (0)
+#else
+#define FAV_STAMP(arr, j, k) do { } while (0)
+#endif
+
 namespace {
 
 constexpr int BM = 128;          // query rows per tile (= TMEM lanes)
 constexpr int BN = 128;          // keys per tile
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
+constexpr int kMmaWarp = 8, kLoadWarp = 9;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleThreshold = 8.0f;   // log2 units: rescale when max grows by > 2^8
 
-template <int D> struct PrefillCfg {
-    static constexpr int kStages = (D == 128) ? 2 : 3;      // K/V ring depth
-    static constexpr int kBoxes = D / 64;
-    static constexpr int kQBytes = BM * D * 2;
-    static constexpr int kKVBytes = BN * D * 2;              // one K or V tile
-    static constexpr int kPBytes = BM * BN * 2;
-    // shared-memory map (offsets from the 1024-aligned base)
-    static constexpr int kOffQ = 0;
-    static constexpr int kOffK = kOffQ + kQBytes;
-    static constexpr int kOffV = kOffK + kStages * kKVBytes;
-    static constexpr int kOffP = kOffV + kStages * kKVBytes;
-    static constexpr int kOnesBytes = 16 * 128;              // 16 rows x 64 ones (bf16)
-    static constexpr int kOffOnes = kOffP + kPBytes;
-    static constexpr int kOffBar = kOffOnes + 1024 * ((kOnesBytes + 1023) / 1024);
-    static constexpr int kNumBars = 1 + 4 * kStages + 2 + 2 + 2;
-    static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
-    static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
-    static constexpr uint32_t kTmemCols = 512;               // S0 | S1 | O
-    static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
-    static constexpr uint32_t kColL = kColO + D;             // 16 columns of sum_k P~[row][k]
-};
+// 2^x for a pair of weights with ex2 on the special-function unit.  (Computing a share of them
+// with a polynomial on the FMA pipe was measured slower on this GPU: the softmax is bound by
+// issue slots and latency, not by the ex2 rate.)
+template <int kPair>
+__device__ __forceinline__ float2 exp2_pair(float2 x) {
+    return make_float2(fav::fast_exp2(x.x), fav::fast_exp2(x.y));
+}
+
+// Calls f(std::integral_constant-like index) for kI = 0 .. kN-1, each a compile-time constant.
+template <int kI, int kN, typename F>
+__device__ __forceinline__ void static_for(F &&f) {
+    if constexpr (kI < kN) {
+        f(std::integral_constant<int, kI>{});
+        static_for<kI + 1, kN>(f);
+    }
+}
 
 template <typename T> struct IsBF16 { static constexpr bool value = false; };
 template <> struct IsBF16<__nv_bfloat16> { static constexpr bool value = true; };
 
-// With bf16 I/O the weights P are rounded to 8 significant bits before the P.V product.  With
-// the lazy maximum a dominant weight can be any value up to 2^8, so normalising the rounded
-// numerator by the unrounded fp32 sum would leave the dominant term off by up to 2^-9 of |v|.
-// The bf16 kernel therefore divides by l~ = sum_k P~[row][k], accumulated by the tensor core
-// (P~ times a column of ones) next to O, so numerator and denominator use the same weights;
-// the fp32 sum of the unrounded weights still gives the LSE.  fp16 keeps 11 bits and divides
-// by the fp32 sum.
-template <typename T> struct RoundedNorm { static constexpr bool value = IsBF16<T>::value; };
+// With bf16 I/O the weights P are split as P = P_hi + P_lo with P_hi = bf16(p) and
+// P_lo = bf16(p - P_hi), and O accumulates P_hi.V + P_lo.V (two MMAs per k-step): together
+// they carry about 16 significant bits of each weight.  With a single bf16 P (8 bits) the
+// weights' rounding alone can move O by up to 2^-9 of |v| when a few weights dominate (any
+// reference maximum, lazy or not, leaves most of them inexact), which with the bf16 rounding
+// of O itself does not fit a 3e-3 error budget.  fp16 keeps 11 bits and uses one MMA.
+template <typename T> struct SplitP { static constexpr bool value = IsBF16<T>::value; };
+
+template <int D> struct PrefillCfg {
+    static constexpr int kStages = (D == 128) ? 2 : 3;      // K/V ring depth
+    static constexpr int kBoxes = D / 64;
+    static constexpr int kQBytes = BM * D * 2;               // one Q tile
+    static constexpr int kKVBytes = BN * D * 2;              // one K or V tile
+    // shared-memory map (offsets from the 1024-aligned base)
+    static constexpr int kOffQ = 0;                          // Q tile 0, Q tile 1
+    static constexpr int kOffK = kOffQ + 2 * kQBytes;
+    static constexpr int kOffV = kOffK + kStages * kKVBytes;
+    static constexpr int kOffBar = kOffV + kStages * kKVBytes;
+    static constexpr int kNumBars = 1 + 4 * kStages + 2 + 2 + 2;
+    static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
+    static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
+    // TMEM columns: S0 | S1 | O0 | O1.  P_i aliases S_i: P_hi in its first 64 columns,
+    // P_lo (bf16 only) in the next 64.
+    static constexpr uint32_t kTmemCols = 512;
+    static __host__ __device__ constexpr uint32_t colS(int i) { return i ? 128u : 0u; }
+    static __host__ __device__ constexpr uint32_t colO(int i) { return 256u + (i ? D : 0); }
+    static_assert(256 + 2 * D <= 512, "TMEM budget");
+};
 
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads, 1)
 fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, T *__restrict__ o,
-                   float *__restrict__ lse, int Hq, int Hkv, int Nq, int Nkv, int n_qtiles,
-                   float scale_log2, int causal, int *status) {
+                   float *__restrict__ lse, int B, int Hq, int Hkv, int Nq, int Nkv,
+                   int n_qtiles, int pair_heads, float scale_log2, int causal, int *status) {
     using C = PrefillCfg<D>;
+    constexpr bool kSplit = SplitP<T>::value;
     constexpr int S = C::kStages;
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment in the shared window (the 128-byte swizzle atom of TMA and MMA)
     const uint32_t raw_u32 = fav::smem_u32(smem_raw);
     uint8_t *smem = smem_raw + ((1024u - (raw_u32 & 1023u)) & 1023u);
     const uint32_t sbase = fav::smem_u32(smem);
-    const uint32_t sQ = sbase + C::kOffQ, sK = sbase + C::kOffK, sV = sbase + C::kOffV;
-    const uint32_t sP = sbase + C::kOffP;
-    // barriers
+    const uint32_t sK = sbase + C::kOffK, sV = sbase + C::kOffV;
     const uint32_t bar0 = sbase + C::kOffBar;
     const uint32_t q_full = bar0;
     const uint32_t k_full = bar0 + 8, k_empty = k_full + 8 * S;
     const uint32_t v_full = k_empty + 8 * S, v_empty = v_full + 8 * S;
-    const uint32_t s_full = v_empty + 8 * S;      // [2]
-    const uint32_t s_free = s_full + 16;          // [2]
-    const uint32_t p_full = s_free + 16;
-    const uint32_t p_empty = p_full + 8;
+    const uint32_t s_full = v_empty + 8 * S;      // [2], one per query tile
+    const uint32_t p_full = s_full + 16;          // [2]
+    const uint32_t o_done = p_full + 16;          // [2]
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffTmemSlot);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int BH = gridDim.x / n_qtiles;
-    const int qtile = n_qtiles - 1 - (int)(blockIdx.x / BH);   // heaviest (causal) tiles first
-    const int bh = blockIdx.x % BH;                            // b * Hq + h
-    const int b = bh / Hq, h = bh % Hq;
     const int G = Hq / Hkv;
-    const int bkv = b * Hkv + h / G;
-    const int q0 = qtile * BM;
-    const int off = Nkv - Nq;                                  // bottom-right causal offset
-    const int kv_end = causal ? min(Nkv, q0 + BM + off) : Nkv; // keys any row of the tile sees
-    const int n_kv = (kv_end + BN - 1) / BN;
 
-    if (warp == 0 && lane == 0) {
+    // ---- the two query tiles of this CTA (heaviest causal work first) ----
+    int b, h[2], t[2];
+    if (pair_heads) {
+        const int units = B * (Hq / 2);
+        const int u = blockIdx.x % units;
+        t[0] = t[1] = n_qtiles - 1 - (int)(blockIdx.x / units);
+        b = u / (Hq / 2);
+        h[0] = 2 * (u % (Hq / 2));
+        h[1] = h[0] + 1;
+    } else {
+        const int BH = B * Hq;
+        const int n_pairs = (n_qtiles + 1) / 2;
+        const int bh = blockIdx.x % BH;
+        const int pr = n_pairs - 1 - (int)(blockIdx.x / BH);
+        b = bh / Hq;
+        h[0] = h[1] = bh % Hq;
+        t[0] = 2 * pr;
+        t[1] = 2 * pr + 1;
+    }
+    const int bkv = b * Hkv + h[0] / G;
+    const int off = Nkv - Nq;                                   // bottom-right causal offset
+    int n_kv_tiles[2];
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        if (t[i] >= n_qtiles) {
+            n_kv_tiles[i] = 0;
+        } else {
+            const int kv_end = causal ? min(Nkv, t[i] * BM + BM + off) : Nkv;
+            n_kv_tiles[i] = (kv_end + BN - 1) / BN;
+        }
+    }
+    const int n_kv = max(n_kv_tiles[0], n_kv_tiles[1]);
+
+    if (warp == kLoadWarp && lane == 0) {
         (void)FAV_CHECK((sbase & 1023u) == 0, status);
         (void)FAV_CHECK((sbase - raw_u32) + C::kOffTmemSlot + 4 <= fav::dynamic_smem_bytes(), status);
         fav::mbar_init(q_full, 1);
@@ -118,21 +178,18 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             fav::mbar_init(v_full + 8 * s, 1);
             fav::mbar_init(v_empty + 8 * s, 1);
         }
-        for (int s = 0; s < 2; ++s) {
-            fav::mbar_init(s_full + 8 * s, 1);
-            fav::mbar_init(s_free + 8 * s, 4);
+        for (int i = 0; i < 2; ++i) {
+            fav::mbar_init(s_full + 8 * i, 1);
+            fav::mbar_init(p_full + 8 * i, 4);
+            fav::mbar_init(o_done + 8 * i, 1);
         }
-        fav::mbar_init(p_full, 4);
-        fav::mbar_init(p_empty, 1);
         fav::mbar_fence_init();
     }
-    if (RoundedNorm<T>::value && warp >= 2) {
-        // bf16 1.0 = 0x3F80; every element of the tile is one, so its layout is irrelevant.
-        uint32_t *ones = reinterpret_cast<uint32_t *>(smem + C::kOffOnes);
-        for (int i = threadIdx.x - 64; i < C::kOnesBytes / 4; i += kThreads - 64) ones[i] = 0x3F803F80u;
-        fav::tc::fence_proxy_async_smem();
-    }
-    if (warp == 1) {
+#ifdef FAV_TIMING
+    __shared__ long long t_ref;
+    if (threadIdx.x == 0) t_ref = clock64();
+#endif
+    if (warp == kMmaWarp) {
         fav::tc::tmem_alloc(fav::smem_u32(tmem_slot), C::kTmemCols);
         fav::tc::tmem_relinquish();
     }
@@ -142,16 +199,23 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     const uint32_t tmem = *tmem_slot;
     (void)FAV_CHECK((tmem & 0xFFFFu) + C::kTmemCols <= 512u && (tmem >> 16) == 0u, status);
 
-    if (warp == 0) {
+    if (warp == kLoadWarp) {
         // ---------------- TMA producer ----------------
         if (lane == 0) {
             fav::tma_prefetch_desc(&tmQ);
             fav::tma_prefetch_desc(&tmK);
             fav::tma_prefetch_desc(&tmV);
-            fav::mbar_arrive_expect_tx(q_full, C::kQBytes);
+            const int nq = (n_kv_tiles[0] > 0) + (n_kv_tiles[1] > 0);
+            fav::mbar_arrive_expect_tx(q_full, nq * C::kQBytes);
 #pragma unroll
-            for (int bx = 0; bx < C::kBoxes; ++bx)
-                fav::tma_load_3d(sQ + bx * BM * 128, &tmQ, q_full, bx * 64, q0, bh);
+            for (int i = 0; i < 2; ++i) {
+                if (n_kv_tiles[i] == 0) continue;
+#pragma unroll
+                for (int bx = 0; bx < C::kBoxes; ++bx)
+                    fav::tma_load_3d(sbase + C::kOffQ + i * C::kQBytes + bx * BM * 128, &tmQ, q_full,
+                                     bx * 64, t[i] * BM, b * Hq + h[i]);
+            }
+            // Each stage has its own empty barriers (one commit per use, waited in order).
             for (int j = 0; j < n_kv; ++j) {
                 const int st = j % S;
                 const uint32_t ph = ((j / S) + 1) & 1;   // parity of the previous use's phase
@@ -169,185 +233,324 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                                      bx * 64, j * BN, bkv);
             }
         }
-    } else if (warp == 1) {
+    } else if (warp == kMmaWarp) {
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
             constexpr bool bf = IsBF16<T>::value;
             constexpr uint32_t idesc_qk = fav::tc::idesc_f16(BM, BN, bf, false);
             constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, bf, true);
-            constexpr uint32_t idesc_l = fav::tc::idesc_f16(BM, 16, bf, false);
-            const uint64_t ones_desc = fav::tc::sdesc_sw128(sbase + C::kOffOnes, 16, 1024);
-            bool ok = fav::mbar_wait(q_full, 0, status);
-            // S_j = Q K_j^T into S buffer j % 2
-            auto issue_s = [&](int j) -> bool {
-                const int st = j % S;
-                if (!fav::mbar_wait(k_full + 8 * st, (j / S) & 1, status)) return false;
-                if (j >= 2 && !fav::mbar_wait(s_free + 8 * (j & 1), ((j >> 1) + 1) & 1, status))
-                    return false;
-                fav::tc::fence_after();
-                const uint32_t d_tmem = tmem + ((j & 1) ? C::kColS1 : C::kColS0);
-                const uint32_t kst = sK + st * C::kKVBytes;
+            // Descriptors are built once; a k-step only adds its byte offset (>> 4) to the
+            // start-address field, which cannot carry out of its 14 bits (addresses < 256 KB).
+            const uint64_t dq0 = fav::tc::sdesc_sw128(sbase + C::kOffQ, 16, 1024);
+            const uint64_t dk0 = fav::tc::sdesc_sw128(sK, 16, 1024);
+            const uint64_t dv0 = fav::tc::sdesc_sw128(sV, BN * 128, 1024);
+            // S_i = Q_i K_j^T
+            auto issue_s = [&](int i, int j) {
+                const uint64_t dq = dq0 + (uint64_t)((i * C::kQBytes) >> 4);
+                const uint64_t dk = dk0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4);
+                const uint32_t d_tmem = tmem + C::colS(i);
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint32_t koff = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
-                    const uint64_t ad = fav::tc::sdesc_sw128(sQ + koff, 16, 1024);
-                    const uint64_t bd = fav::tc::sdesc_sw128(kst + (kk >> 2) * (BN * 128) + (kk & 3) * 32,
-                                                             16, 1024);
-                    fav::tc::mma_ss(d_tmem, ad, bd, idesc_qk, kk > 0);
+                    const uint64_t koff = (uint64_t)((((kk >> 2) * (BM * 128)) + (kk & 3) * 32) >> 4);
+                    fav::tc::mma_ss(d_tmem, dq + koff, dk + koff, idesc_qk, kk > 0);
                 }
-                fav::tc::commit(s_full + 8 * (j & 1));
-                fav::tc::commit(k_empty + 8 * st);
-                return true;
             };
-            if (ok && n_kv > 0) ok = issue_s(0);
-            for (int j = 0; ok && j < n_kv; ++j) {
-                if (j + 1 < n_kv && !issue_s(j + 1)) { ok = false; break; }
-                const int st = j % S;
-                if (!fav::mbar_wait(p_full, j & 1, status)) { ok = false; break; }
-                if (!fav::mbar_wait(v_full + 8 * st, (j / S) & 1, status)) { ok = false; break; }
-                fav::tc::fence_after();
-                const uint32_t vst = sV + st * C::kKVBytes;
+            // O_i += P_i V_j, with P_i read from TMEM (8 columns = 16 keys per k-step; bf16 adds
+            // P_lo from 64 columns further) and V MN-major in shared memory (8-key groups
+            // 1024 B apart, 64-column blocks one box apart).
+            auto issue_pv = [&](int i, int j) {
+                const uint64_t dv = dv0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4);
+                const uint32_t s_tmem = tmem + C::colS(i);
+                const uint32_t o_tmem = tmem + C::colO(i);
+                const uint32_t acc = (j > 0) ? 1u : 0u;
 #pragma unroll
                 for (int kk = 0; kk < BN / 16; ++kk) {
-                    // A = P (128 rows x 16 keys, K-major); B = V (16 keys x D, MN-major:
-                    // 8-key groups 1024 B apart, 64-column blocks one TMA box apart).
-                    const uint64_t ad = fav::tc::sdesc_sw128(
-                        sP + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
-                    const uint64_t bd = fav::tc::sdesc_sw128(vst + kk * 16 * 128, BN * 128, 1024);
-                    fav::tc::mma_ss(tmem + C::kColO, ad, bd, idesc_pv, (j > 0 || kk > 0));
-                    if (RoundedNorm<T>::value)
-                        fav::tc::mma_ss(tmem + C::kColL, ad, ones_desc, idesc_l, (j > 0 || kk > 0));
+                    const uint64_t bd = dv + (uint64_t)((kk * 16 * 128) >> 4);
+                    fav::tc::mma_ts(o_tmem, s_tmem + kk * 8, bd, idesc_pv, acc | (kk > 0));
+                    if (kSplit) fav::tc::mma_ts(o_tmem, s_tmem + 64 + kk * 8, bd, idesc_pv, 1u);
                 }
-                fav::tc::commit(v_empty + 8 * st);
-                fav::tc::commit(p_empty);
+            };
+#ifdef FAV_TIMING
+            long long ts[16][6];
+            const long long t_start = t_ref;
+#endif
+            bool ok = fav::mbar_wait(q_full, 0, status) && fav::mbar_wait(k_full, 0, status);
+            if (ok) {
+                fav::tc::fence_after();
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (n_kv_tiles[i] == 0) continue;
+                    issue_s(i, 0);
+                    fav::tc::commit(s_full + 8 * i);
+                }
+                fav::tc::commit(k_empty);
             }
+            // Issue order per key tile j: [P_0(j).V_j, S_0(j+1)], [P_1(j).V_j, S_1(j+1)]: the
+            // scores of the two tiles arrive half a period apart, so each softmax runs while the
+            // tensor core works on the other tile.
+            for (int j = 0; ok && j < n_kv; ++j) {
+                const int st = j % S, st1 = (j + 1) % S;
+                const bool nxt = j + 1 < n_kv;
+                // tested ahead: V_j now, K_{j+1} before the first burst, P_1(j) before the second
+                bool v_ready = fav::mbar_try(v_full + 8 * st, (j / S) & 1);
+                bool k_ready = !nxt;
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (j >= n_kv_tiles[i]) continue;
+                    FAV_STAMP(ts, j, 3 * i);
+                    if (!fav::mbar_wait_fast(p_full + 8 * i, j & 1, status)) { ok = false; break; }
+                    if (!v_ready) {
+                        if (!fav::mbar_wait(v_full + 8 * st, (j / S) & 1, status)) { ok = false; break; }
+                        v_ready = true;
+                    }
+                    FAV_STAMP(ts, j, 3 * i + 1);
+                    fav::tc::fence_after();
+                    const bool k_tested = k_ready || fav::mbar_try(k_full + 8 * st1, ((j + 1) / S) & 1);
+                    issue_pv(i, j);
+                    if (j + 1 < n_kv_tiles[i]) {
+                        if (!k_tested && !fav::mbar_wait(k_full + 8 * st1, ((j + 1) / S) & 1, status)) {
+                            ok = false;
+                            break;
+                        }
+                        k_ready = true;
+                        fav::tc::fence_after();
+                        issue_s(i, j + 1);
+                        fav::tc::commit(s_full + 8 * i);
+                    } else {
+                        fav::tc::commit(o_done + 8 * i);
+                    }
+                    FAV_STAMP(ts, j, 3 * i + 2);
+                }
+                if (!ok) break;
+                fav::tc::commit(v_empty + 8 * st);
+                if (nxt) fav::tc::commit(k_empty + 8 * st1);
+            }
+#ifdef FAV_TIMING
+            if (blockIdx.x == 0)
+                for (int j = 0; j < min(n_kv, 16); ++j)
+                    printf("[mma] j=%2d wait_p0 %6lld got_p0 %6lld done0 %6lld | wait_p1 %6lld got_p1 %6lld done1 %6lld\n", j,
+                           ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start, ts[j][3] - t_start,
+                           ts[j][4] - t_start, ts[j][5] - t_start);
+#endif
         }
     } else {
-        // ---------------- softmax / correction / epilogue (one thread per row) ----------------
+        // ---------------- softmax / correction / epilogue: one thread per query row ----------------
+        const int i = warp >> 2;                          // query tile of this warpgroup
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;
+        const int ti = i ? t[1] : t[0];
+        const int hi = i ? h[1] : h[0];
+        const int q0 = ti * BM;
         const int qi = q0 + row;                          // query index of this row
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
-        const int lim = causal ? min(Nkv, qi + off + 1) : Nkv;   // visible keys: [0, lim)
-        const int lim_tile = causal ? min(Nkv, q0 + off + 1) : Nkv;  // smallest lim in tile
+        const uint32_t colS = i ? C::colS(1) : C::colS(0);
+        const uint32_t colO = i ? C::colO(1) : C::colO(0);
+        const int lim = causal ? min(Nkv, qi + off + 1) : Nkv;       // visible keys: [0, lim)
+        const int lim_tile = causal ? min(Nkv, q0 + off + 1) : Nkv;  // smallest lim in the tile
+        const int n_mine = i ? n_kv_tiles[1] : n_kv_tiles[0];
         float m = -INFINITY, l = 0.f;
         bool ok = true;
-        for (int j = 0; j < n_kv; ++j) {
-            const uint32_t sb = j & 1;
-            if (!fav::mbar_wait(s_full + 8 * sb, (j >> 1) & 1, status)) { ok = false; break; }
+#ifdef FAV_TIMING
+        long long ts[16][6];
+        const long long t_start = t_ref;
+#endif
+        for (int j = 0; j < n_mine; ++j) {
+            FAV_STAMP(ts, j, 0);
+            if (!fav::mbar_wait(s_full + 8 * i, j & 1, status)) { ok = false; break; }
+            FAV_STAMP(ts, j, 1);
             fav::tc::fence_after();
-            float s[BN];
-            {
-                const uint32_t scol = trow + (sb ? C::kColS1 : C::kColS0);
-#pragma unroll
-                for (int c = 0; c < BN / 32; ++c) {
-                    uint32_t r[32];
-                    fav::tc::ld_32x32b_x32(scol + c * 32, r);
-                    fav::tc::wait_ld();
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(r[e]);
-                }
-            }
-            fav::tc::fence_before();
-            __syncwarp();
-            if (lane == 0) fav::mbar_arrive(s_free + 8 * sb);
-
             const int key0 = j * BN;
-            if (key0 + BN > lim_tile) {     // tile crosses the causal diagonal or the end
+            const bool crosses = key0 + BN > lim_tile;   // tile crosses the diagonal or the end
+            float s[BN];
+            // S row from TMEM (and the mask: keys at or beyond lim get -inf)
+            auto load_s = [&]() {
+                uint32_t r[BN / 32][32];
 #pragma unroll
-                for (int c = 0; c < BN; ++c)
-                    if (key0 + c >= lim) s[c] = -INFINITY;
-            }
-            float mx = s[0];
+                for (int c = 0; c < BN / 32; ++c) fav::tc::ld_32x32b_x32(trow + colS + c * 32, r[c]);
 #pragma unroll
-            for (int c = 1; c < BN; ++c) mx = fmaxf(mx, s[c]);
-            mx *= scale_log2;
-            // lazy rescale: move the reference maximum only when it grows by > 2^8
+                for (int c = 0; c < BN / 32; ++c) fav::tc::wait_ld_dep(r[c]);
+#pragma unroll
+                for (int c = 0; c < BN; ++c) s[c] = __uint_as_float(r[c >> 5][c & 31]);
+                if (crosses) {
+#pragma unroll
+                    for (int c = 0; c < BN; ++c)
+                        if (key0 + c >= lim) s[c] = -INFINITY;
+                }
+            };
+            // raw row maximum: 8 independent chains of 3-input max, then a tree
+            auto row_max = [&]() {
+                float m8[8];
+#pragma unroll
+                for (int c = 0; c < 8; ++c) m8[c] = s[c];
+#pragma unroll
+                for (int c = 8; c < BN; c += 16) {
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) m8[k] = fav::fmax3(m8[k], s[c + k], s[c + 8 + k]);
+                }
+                return fav::fmax3(fav::fmax3(m8[0], m8[1], m8[2]), fav::fmax3(m8[3], m8[4], m8[5]),
+                                  fmaxf(m8[6], m8[7]));
+            };
+            // p = exp2(s * scale_log2 - mref) on pairs (one packed FMA, two ex2, one packed
+            // add): packed weights, their fp32 sum, and the raw row maximum of the same pass.
+            uint32_t pk[2][32];
+            float psum = 0.f;
+            auto exp_pass = [&](float mref) {
+                const float2 sc2 = make_float2(scale_log2, scale_log2);
+                const float2 nm2 = make_float2(-mref, -mref);
+                float2 l4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                static_for<0, BN / 2>([&](auto pc) {
+                    constexpr int c = 2 * decltype(pc)::value;
+                    const float2 x = fav::ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
+                    const float2 p = exp2_pair<c / 2>(x);
+                    l4[(c >> 1) & 3] = fav::fadd2(l4[(c >> 1) & 3], p);
+                    m4[(c >> 1) & 3] = fav::fmax3(m4[(c >> 1) & 3], s[c], s[c + 1]);
+                    pk[c >> 6][(c >> 1) & 31] = fav::Elem<T>::pack(p.x, p.y);
+                });
+                const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
+                psum = a.x + a.y;
+                return fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+            };
+            // bf16: exponentials of keys [64h, 64h + 64) into hi / lo parts, stored to TMEM at
+            // once (P_hi over S columns [32h, 32h + 32), P_lo over [64 + 32h, 96 + 32h)).
+            auto exp_half_store = [&](float mref, int h) {
+                const float2 sc2 = make_float2(scale_log2, scale_log2);
+                const float2 nm2 = make_float2(-mref, -mref);
+                float2 l4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+                uint32_t hi32[32], lo32[32];
+                static_for<0, 32>([&](auto pe) {
+                    constexpr int e = 2 * decltype(pe)::value;
+                    const int c = 64 * h + e;
+                    const float2 x = fav::ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
+                    const float2 p = exp2_pair<e / 2>(x);
+                    l4[(e >> 1) & 3] = fav::fadd2(l4[(e >> 1) & 3], p);
+                    const uint32_t hi = fav::Elem<T>::pack(p.x, p.y);
+                    const float2 hf = make_float2(__uint_as_float(hi << 16), __uint_as_float(hi & 0xFFFF0000u));
+                    const float2 lo = fav::ffma2(hf, make_float2(-1.f, -1.f), p);
+                    hi32[e >> 1] = hi;
+                    lo32[e >> 1] = fav::Elem<T>::pack(lo.x, lo.y);
+                });
+                fav::tc::st_32x32b_x32(trow + colS + 32 * h, hi32);
+                fav::tc::st_32x32b_x32(trow + colS + 64 + 32 * h, lo32);
+                const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
+                psum += a.x + a.y;
+            };
             float alpha = 1.f;
             bool rescale = false;
-            if (mx > m + kRescaleThreshold) {
-                alpha = fav::fast_exp2(m - mx);       // 0 on the first tile (m = -inf)
-                rescale = (j > 0);
-                m = mx;
-                l *= alpha;
-            }
-            uint32_t pk[BN / 2];
-            const float neg_m = -m;
-#pragma unroll
-            for (int c = 0; c < BN; c += 2) {
-                const float p0 = fav::fast_exp2(fmaf(s[c], scale_log2, neg_m));
-                const float p1 = fav::fast_exp2(fmaf(s[c + 1], scale_log2, neg_m));
-                l += p0 + p1;
-                pk[c / 2] = fav::Elem<T>::pack(p0, p1);
-            }
-            // PV_{j-1} must be done: it reads the P buffer and accumulates into O.
-            if (j > 0 && !fav::mbar_wait(p_empty, (j - 1) & 1, status)) { ok = false; break; }
-            fav::tc::fence_after();
-            if (__any_sync(~0u, rescale)) {
-                constexpr int kChunks = D / 32 + (RoundedNorm<T>::value ? 1 : 0);   // O (+ l~)
-#pragma unroll
-                for (int c = 0; c < kChunks; ++c) {
-                    uint32_t r[32];
-                    fav::tc::ld_32x32b_x32(trow + C::kColO + c * 32, r);
-                    fav::tc::wait_ld();
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-                    fav::tc::st_32x32b_x32(trow + C::kColO + c * 32, r);
+            // lazy rescale: move the reference maximum only when it grows by > 2^8
+            auto move_max = [&](float mx) {
+                if (mx > m + kRescaleThreshold) {
+                    alpha = fav::fast_exp2(m - mx);   // 0 on the first tile (m = -inf)
+                    rescale = (j > 0);
+                    m = mx;
+                    l *= alpha;
                 }
-                fav::tc::wait_st();
+            };
+            if constexpr (kSplit) {
+                // two passes: the row maximum first, then the weights, stored as produced
+                load_s();
+                FAV_STAMP(ts, j, 2);
+                move_max(row_max() * scale_log2);
+                FAV_STAMP(ts, j, 3);
+                psum = 0.f;
+                exp_half_store(m, 0);
+                exp_half_store(m, 1);
+            } else if (j == 0) {
+                load_s();
+                FAV_STAMP(ts, j, 2);
+                move_max(row_max() * scale_log2);
+                FAV_STAMP(ts, j, 3);
+                exp_pass(m);
+            } else {
+                // After the first tile the weights are computed speculatively against the
+                // current reference maximum while the tile's own maximum is found in the same
+                // pass; a warp with a row whose maximum grew by more than 2^8 (rare) reloads
+                // the scores and redoes the tile (warp-uniform: tcgen05.ld is collective).
+                load_s();
+                FAV_STAMP(ts, j, 2);
+                const bool redo = exp_pass(m) * scale_log2 > m + kRescaleThreshold;
+                FAV_STAMP(ts, j, 3);
+                if (__any_sync(~0u, redo)) {
+                    load_s();
+                    move_max(row_max() * scale_log2);
+                    exp_pass(m);
+                }
             }
-            // P row -> shared memory, K-major, 128-byte swizzle (two 64-key blocks).
+            l += psum;
+            FAV_STAMP(ts, j, 4);
+            // (after the exponentials, so that only the packed weights are live)
+            // O_i is stable here: P_i(j-1).V completed before S_i(j) (in-order MMAs, one commit).
+            if (__any_sync(~0u, rescale)) {
 #pragma unroll
-            for (int cc = 0; cc < BN / 8; ++cc) {
-                const uint32_t addr = sP + (cc >> 3) * (BM * 128) + row * 128 +
-                                      ((((uint32_t)cc & 7u) ^ ((uint32_t)row & 7u)) << 4);
-                if (!FAV_CHECK(addr >= sP && addr + 16 <= sP + C::kPBytes, status)) continue;
-                asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};"
-                             ::"r"(addr), "r"(pk[4 * cc]), "r"(pk[4 * cc + 1]), "r"(pk[4 * cc + 2]),
-                               "r"(pk[4 * cc + 3]) : "memory");
+                for (int c = 0; c < D / 32; ++c) {
+                    const uint32_t col = colO + c * 32;
+                    uint32_t v[32];
+                    fav::tc::ld_32x32b_x32(trow + col, v);
+                    fav::tc::wait_ld_dep(v);
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        const float2 y = fav::fmul2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])),
+                                                    make_float2(alpha, alpha));
+                        v[e] = __float_as_uint(y.x);
+                        v[e + 1] = __float_as_uint(y.y);
+                    }
+                    fav::tc::st_32x32b_x32(trow + col, v);
+                }
             }
-            fav::tc::fence_proxy_async_smem();
+            // P_i over the first 64 columns of S_i (two 16-bit weights per column); bf16 has
+            // stored its hi and lo parts already.
+            if constexpr (!kSplit) {
+                fav::tc::st_32x32b_x32(trow + colS, pk[0]);
+                fav::tc::st_32x32b_x32(trow + colS + 32, pk[1]);
+            }
+            fav::tc::wait_st();
             fav::tc::fence_before();
             __syncwarp();
-            if (lane == 0) fav::mbar_arrive(p_full);
+            if (lane == 0) fav::mbar_arrive(p_full + 8 * i);
+            FAV_STAMP(ts, j, 5);
         }
+#ifdef FAV_TIMING
+        if (blockIdx.x == 0 && lane == 0 && n_mine > 5)
+            printf("[w%d j5] wait %6lld s_ready %6lld ld %6lld spec %6lld chk %6lld arrive %6lld\n", warp,
+                   ts[5][0] - t_start, ts[5][1] - t_start, ts[5][2] - t_start, ts[5][3] - t_start,
+                   ts[5][4] - t_start, ts[5][5] - t_start);
+        if (blockIdx.x == 0 && (threadIdx.x & 127) == 0)
+            for (int j = 0; j < min(n_mine, 16); ++j)
+                printf("[sm%d] j=%2d wait %6lld s_ready %6lld ld %6lld max %6lld exp %6lld arrive %6lld\n",
+                       i, j, ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start,
+                       ts[j][3] - t_start, ts[j][4] - t_start, ts[j][5] - t_start);
+#endif
         // ---------------- epilogue: O / l, LSE ----------------
-        if (ok && n_kv > 0 && fav::mbar_wait(p_empty, (n_kv - 1) & 1, status)) {
+        if (ok && n_mine > 0 && fav::mbar_wait(o_done + 8 * i, 0, status)) {
             fav::tc::fence_after();
-            float inv_l = 1.f / l;
-            if (RoundedNorm<T>::value) {
-                uint32_t r[32];
-                fav::tc::ld_32x32b_x32(trow + C::kColL, r);
-                fav::tc::wait_ld();
-                inv_l = 1.f / __uint_as_float(r[0]);
-            }
+            const float inv_l = 1.f / l;
             const bool valid = qi < Nq;
-            T *orow = o + ((long long)bh * Nq + qi) * D;
+            T *orow = o + ((long long)(b * Hq + hi) * Nq + qi) * D;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
-                uint32_t r[32];
-                fav::tc::ld_32x32b_x32(trow + C::kColO + c * 32, r);
-                fav::tc::wait_ld();
+                uint32_t v[32];
+                fav::tc::ld_32x32b_x32(trow + colO + c * 32, v);
+                fav::tc::wait_ld_dep(v);
                 if (valid) {
 #pragma unroll
                     for (int e = 0; e < 32; e += 8) {
                         uint4 v4;
-                        v4.x = fav::Elem<T>::pack(__uint_as_float(r[e]) * inv_l, __uint_as_float(r[e + 1]) * inv_l);
-                        v4.y = fav::Elem<T>::pack(__uint_as_float(r[e + 2]) * inv_l, __uint_as_float(r[e + 3]) * inv_l);
-                        v4.z = fav::Elem<T>::pack(__uint_as_float(r[e + 4]) * inv_l, __uint_as_float(r[e + 5]) * inv_l);
-                        v4.w = fav::Elem<T>::pack(__uint_as_float(r[e + 6]) * inv_l, __uint_as_float(r[e + 7]) * inv_l);
+                        v4.x = fav::Elem<T>::pack(__uint_as_float(v[e]) * inv_l, __uint_as_float(v[e + 1]) * inv_l);
+                        v4.y = fav::Elem<T>::pack(__uint_as_float(v[e + 2]) * inv_l, __uint_as_float(v[e + 3]) * inv_l);
+                        v4.z = fav::Elem<T>::pack(__uint_as_float(v[e + 4]) * inv_l, __uint_as_float(v[e + 5]) * inv_l);
+                        v4.w = fav::Elem<T>::pack(__uint_as_float(v[e + 6]) * inv_l, __uint_as_float(v[e + 7]) * inv_l);
                         *reinterpret_cast<uint4 *>(orow + c * 32 + e) = v4;
                     }
                 }
             }
-            if (valid && lse) lse[(long long)bh * Nq + qi] = (m + log2f(l)) * kLn2;
+            if (valid && lse) lse[(long long)(b * Hq + hi) * Nq + qi] = (m + log2f(l)) * kLn2;
         }
     }
 
     fav::tc::fence_before();
     __syncthreads();
     fav::tc::fence_after();
-    if (warp == 1) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
+    if (warp == kMmaWarp) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
 }
 
 template <typename T, int D>
@@ -363,11 +566,14 @@ fav_status launch(const FavArgs &a, cudaStream_t stream) {
         cudaSuccess)
         return FAV_ERR_CUDA;
     const int n_qtiles = (a.Nq + BM - 1) / BM;
-    const long long blocks = (long long)n_qtiles * a.B * a.Hq;
+    const int G = a.Hq / a.Hkv;
+    const int pair_heads = (G % 2 == 0) ? 1 : 0;
+    const long long blocks = pair_heads ? (long long)n_qtiles * a.B * (a.Hq / 2)
+                                        : (long long)((n_qtiles + 1) / 2) * a.B * a.Hq;
     if (blocks > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
     kern<<<(unsigned)blocks, kThreads, C::kSmemBytes, stream>>>(
-        tmQ, tmK, tmV, (T *)a.o, a.lse, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles, a.scale * kLog2e,
-        a.causal, a.dev_status);
+        tmQ, tmK, tmV, (T *)a.o, a.lse, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles, pair_heads,
+        a.scale * kLog2e, a.causal, a.dev_status);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_kernel", stream))
         return FAV_ERR_CUDA;
     return FAV_OK;

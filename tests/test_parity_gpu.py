@@ -144,3 +144,41 @@ def test_error_leaves_outputs_untouched():
         fav.forward(q, k, k, out=o)
     torch.cuda.synchronize()
     assert bool((o == 7.0).all())
+
+
+# ---- prefill path edge cases ----
+
+@pytest.mark.parametrize("dtype,D,causal", [(I.F16, 128, True), (I.BF16, 64, True),
+                                            (I.BF16, 128, False), (I.F16, 64, False)])
+def test_prefill_growing_scores(dtype, D, causal):
+    """Keys scaled by a ramp along the sequence: the row maximum keeps growing from tile to
+    tile, so the lazy rescale and the speculative-exponential redo both run many times."""
+    w = W(dtype, 1, 4, 2, 700, 700, D, causal=causal, seed=40 + D)
+    x = I.make_inputs(w)
+    ramp = np.linspace(1.0, 12.0, w.Nkv)[None, None, :, None]
+    k = I.round_to_dtype(x["k"] * ramp, dtype)
+    x = dict(x, k=k, k_bits=I.to_storage(k, dtype))
+    fav.set_path(fav.PATH_PREFILL)
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_PREFILL
+    check(w, o, lse, x)
+
+
+@pytest.mark.parametrize("Nq,Nkv,causal", [(1, 1, False), (5, 5, True), (128, 128, True),
+                                           (129, 129, True), (255, 1000, True), (300, 40, False)])
+def test_prefill_ragged_shapes(Nq, Nkv, causal):
+    fav.set_path(fav.PATH_PREFILL)
+    w = W(I.BF16, 1, 2, 1, Nq, Nkv, 128, causal=causal, seed=Nq + Nkv)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    check(w, o, lse, x)
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(3, 1), (6, 3), (5, 5), (8, 1)])
+def test_prefill_head_pairings(Hq, Hkv):
+    """Even groups pair two heads per block; odd groups pair two query tiles of one head."""
+    fav.set_path(fav.PATH_PREFILL)
+    w = W(I.F16, 2, Hq, Hkv, 260, 260, 64, causal=True, seed=Hq * 7 + Hkv)
+    x = I.make_inputs(w)
+    o, lse = run_gpu(w, x)
+    check(w, o, lse, x)
