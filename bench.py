@@ -8,8 +8,8 @@ The same JSON line also reports the other workloads of the measurement plan (GQA
 prefill with outliers; fp16 GQA and bf16 MQA decode with the split-KV combine, in KV GB/s).
 
 Timing: W warm-up steps, then K timed steps, each bracketed by CUDA events on the launching
-stream; L2 is flushed before every timed step by writing a 256 MiB buffer (outside the
-events).  e2e = the same metric through the host-buffer C-ABI call fav_forward_host
+stream; L2 is flushed before every timed step by reading a 256 MiB buffer (outside the
+events; a read leaves no dirty lines whose write-back would compete with the timed kernel).  e2e = the same metric through the host-buffer C-ABI call fav_forward_host
 (pinned host inputs copied in, O and LSE copied out, every step).  cpu_baseline = the fp64
 oracle on the host cores on a bounded sample of the workload (rank 0, N=1 only).
 --impl reference times that oracle as the reference arm.
@@ -168,9 +168,15 @@ def launches_per_call(fav):
 
 
 def time_device(fn, steps, warmup, stream, dist):
-    """Per-step CUDA-event times (ms) of `fn`, L2 flushed before each timed step."""
+    """Per-step CUDA-event times (ms) of `fn`, L2 flushed before each timed step.
+
+    The flush READS a 256 MiB buffer (twice the L2): it evicts the previous step's data and
+    leaves only clean lines behind.  (A write-based flush would leave ~126 MB of dirty lines
+    whose write-back then competes with the timed kernel's own HBM traffic.)
+    """
     import torch
-    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
+    flush = torch.ones(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
+    sink = torch.empty((), dtype=torch.uint8, device="cuda")
     for _ in range(warmup):
         fn()
     torch.cuda.synchronize()
@@ -181,7 +187,7 @@ def time_device(fn, steps, warmup, stream, dist):
     t0 = time.perf_counter()
     with torch.cuda.stream(stream):
         for s, e in ev:
-            flush.zero_()
+            torch.amax(flush, dim=0, out=sink)
             s.record(stream)
             fn()
             e.record(stream)
@@ -351,7 +357,7 @@ def fav_arm(args, dist):
         "data": "synthetic (seeded N(0,1) Q/K, U(-1,1) V)",
         "config": {"workload": w.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv, "Nq": w.Nq,
                    "Nkv": w.Nkv, "D": w.D, "causal": w.causal, "path": path,
-                   "l2": "flushed before every timed step (256 MiB write)",
+                   "l2": "flushed before every timed step (256 MiB read, outside the events)",
                    "parallelism": "replicas" if dist.world > 1 else "single GPU"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": pk["tflops"],
                      "unit": "TFLOP/s", "frac": achieved / pk["tflops"], "traffic": traffic,

@@ -26,18 +26,20 @@
 
 namespace {
 
-constexpr int TK = 32;            // keys per tile
-constexpr int kConsumers = 4;     // consumer warps
+constexpr int kConsumers = 6;     // consumer warps
 constexpr int kThreads = (kConsumers + 1) * 32;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
 
-// Ring of kStages stages; tile lt goes to stage lt % kStages and to consumer warp lt % 4.
-// kStages is a multiple of the number of consumer warps, so each stage (and its pair of
-// barriers) belongs to exactly one warp, which waits on its phases strictly in order: a
-// warp can never be two phases behind a barrier it polls (parity would alias).
+// Ring of kStages stages; tile lt goes to stage lt % kStages and to consumer warp
+// lt % kConsumers.  kStages is a multiple of the number of consumer warps, so each stage (and
+// its pair of barriers) belongs to exactly one warp, which waits on its phases strictly in
+// order: a warp can never be two phases behind a barrier it polls (parity would alias).  Two
+// stages per warp let a warp compute on one tile while its next tile is loading; 12 stages of
+// 16 KB keep ~192 KB of K/V reads in flight per SM (one block per SM).
 template <int D> struct DecodeCfg {
-    static constexpr int kStagesPerWarp = (D == 128) ? 1 : 2;
+    static constexpr int TK = (D == 128) ? 32 : 64;           // keys per tile
+    static constexpr int kStagesPerWarp = 2;
     static constexpr int kStages = kConsumers * kStagesPerWarp;
     static constexpr int kBoxes = D / 64;                     // 64-element (128 B) boxes per row
     static constexpr int kTileBytes = TK * D * 2;             // one K (or V) tile
@@ -51,12 +53,13 @@ template <int D> struct DecodeCfg {
 
 // Byte offset of 16-byte chunk `c` (of D/8) in key row `j` of a tile written by TMA with
 // 128-byte swizzle: boxes of 64 elements, each TK rows of 128 B; chunk index XOR (row % 8).
+template <int TK>
 __device__ __forceinline__ uint32_t swz(int j, int c) {
     return (uint32_t)((c >> 3) * (TK * 128) + j * 128 + (((c & 7) ^ (j & 7)) << 4));
 }
 
 template <typename T, int D>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 1)
 fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                   const T *__restrict__ q, T *__restrict__ o, float *__restrict__ lse,
                   float *__restrict__ part_o, float *__restrict__ part_lse, int Hq, int Hkv,
@@ -64,6 +67,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
                   float scale_log2, int causal, int *status) {
     using Cfg = DecodeCfg<D>;
     constexpr int S = Cfg::kStages;
+    constexpr int TK = Cfg::TK;
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment of the ring in the shared window (the 128-byte swizzle atom)
     const uint32_t raw_u32 = fav::smem_u32(smem_raw);
@@ -96,6 +100,15 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     }
     __syncthreads();
 
+#ifdef FAV_TIMING
+    __shared__ long long t_ref;
+    __shared__ long long t_issue[64], t_ready[64], t_done[64];
+    if (threadIdx.x == 0) t_ref = clock64();
+    __syncthreads();
+#define FAV_DSTAMP(arr, lt) do { if ((lt) < 64) arr[lt] = clock64() - t_ref; } while (0)
+#else
+#define FAV_DSTAMP(arr, lt) do { } while (0)
+#endif
     if (warp == kConsumers) {
         // ---------------- producer: one lane streams K/V tiles with TMA ----------------
         if (lane == 0) {
@@ -105,6 +118,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
                 const int st = lt % S;
                 if (lt >= S && !fav::mbar_wait(empty0 + 8 * st, ((lt / S) - 1) & 1, status)) break;
                 const uint32_t full = full0 + 8 * st;
+                FAV_DSTAMP(t_issue, lt);
                 fav::mbar_arrive_expect_tx(full, Cfg::kStageBytes);
                 const int key0 = (tile0 + lt) * TK;
                 const uint32_t kdst = ring_u32 + st * Cfg::kStageBytes;
@@ -165,6 +179,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     for (int lt = warp; lt < my_tiles; lt += kConsumers) {
         const int st = lt % S;
         if (!fav::mbar_wait(full0 + 8 * st, (lt / S) & 1, status)) { ok = false; break; }
+        if (lane == 0) FAV_DSTAMP(t_ready, lt);
         const uint32_t kbase = ring_u32 + st * Cfg::kStageBytes;
         const uint32_t vbase = kbase + Cfg::kTileBytes;
         const int key0 = (tile0 + lt) * TK;
@@ -178,7 +193,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
 #pragma unroll
             for (int nt = 0; nt < TK / 8; ++nt) {
                 uint32_t bfr[4] = {0u, 0u, 0u, 0u};
-                const uint32_t la = kbase + swz(8 * nt + (lane & 7), 4 * kp + (lane >> 3));
+                const uint32_t la = kbase + swz<TK>(8 * nt + (lane & 7), 4 * kp + (lane >> 3));
                 if (FAV_CHECK(la >= ring_u32 && la + 16 <= vbase && (la & 15u) == 0, status))
                     fav::ldmatrix_x4(bfr, la);
                 fav::mma16816<T>(s[nt], qa[2 * kp], bfr[0], bfr[1]);
@@ -241,7 +256,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
 #pragma unroll
             for (int np = 0; np < D / 16; ++np) {
                 uint32_t bfr[4] = {0u, 0u, 0u, 0u};
-                const uint32_t la = vbase + swz(krow, 2 * np + (i4 >> 1));
+                const uint32_t la = vbase + swz<TK>(krow, 2 * np + (i4 >> 1));
                 if (FAV_CHECK(la >= vbase && la + 16 <= ring_u32 + Cfg::kRingBytes && (la & 15u) == 0, status))
                     fav::ldmatrix_x4_trans(bfr, la);
                 fav::mma16816<T>(acc[2 * np], pa, bfr[0], bfr[1]);
@@ -250,6 +265,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         }
         __syncwarp();
         if (lane == 0) fav::mbar_arrive(empty0 + 8 * st);
+        if (lane == 0) FAV_DSTAMP(t_done, lt);
     }
 
     // ---------------- merge the four warp states through shared memory ----------------
@@ -276,9 +292,15 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         redl[warp * 16 + r + 8] = lrow[1];
     }
     fav::named_bar_sync(1, kConsumers * 32);
+#ifdef FAV_TIMING
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0)
+        for (int lt = 0; lt < min(my_tiles, 64); ++lt)
+            printf("[dec] tile %2d issue %7lld ready %7lld done %7lld\n", lt, t_issue[lt], t_ready[lt], t_done[lt]);
+#endif
     if (!ok) return;
 
     constexpr int kCols = D / 8;                 // columns per thread (8 threads per row)
+    if (threadIdx.x >= 128) return;              // 16 rows x 8 threads merge the warps
     const int rr = threadIdx.x >> 3;             // 0..15
     const int c0 = (threadIdx.x & 7) * kCols;
     const int m = m0 + rr;
@@ -400,6 +422,7 @@ fav_combine_kernel(const float *__restrict__ part_o, const float *__restrict__ p
 template <typename T, int D>
 fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t stream) {
     using Cfg = DecodeCfg<D>;
+    constexpr int TK = Cfg::TK;
     alignas(64) CUtensorMap tmK, tmV;
     const int outer = a.B * a.Hkv;
     fav_status st = fav_make_tmap_3d(&tmK, a.k, D, a.Nkv, outer, TK);
@@ -460,16 +483,24 @@ bool fav_decode_supported(const FavArgs &a) {
     return M <= 64 && (long long)a.B * a.Hkv <= 65535;
 }
 
-int fav_decode_num_tiles(const FavArgs &a) { return (a.Nkv + TK - 1) / TK; }
+int fav_decode_num_tiles(const FavArgs &a) {
+    const int tk = (a.D == 128) ? DecodeCfg<128>::TK : DecodeCfg<64>::TK;
+    return (a.Nkv + tk - 1) / tk;
+}
 
-// Enough blocks for several waves of two resident blocks per SM, at least two tiles each.
+// Split count: a single wave of blocks covering ~90% of the SMs.  A block streams its whole
+// key range through the ring, and ~0.9 x SMs streaming blocks already saturate HBM, while
+// every extra block (a second wave, or a partly filled one) adds a ring fill and a final merge
+// to the critical path; measured on the decode workloads, one wave of ~128-144 blocks beat
+// three waves by 10-15%.  Each block keeps at least two tiles per ring stage.
 int fav_decode_auto_splits(const FavArgs &a) {
     const int n_tiles = fav_decode_num_tiles(a);
     const long long M = (long long)a.Nq * (a.Hq / a.Hkv);
     const long long groups = (long long)a.B * a.Hkv * ((M + 15) / 16);
-    const long long target = 8LL * (a.num_sms > 0 ? a.num_sms : 148);
-    long long splits = (target + groups - 1) / groups;
-    splits = std::min<long long>(splits, std::max(1, n_tiles / 2));
+    const long long sms = a.num_sms > 0 ? a.num_sms : 148;
+    long long splits = (9 * sms) / (10 * groups);
+    const int min_tiles = 2 * DecodeCfg<128>::kStages;
+    splits = std::min<long long>(splits, std::max(1, n_tiles / min_tiles));
     splits = std::max<long long>(1, std::min<long long>(splits, 4096));
     return (int)splits;
 }
