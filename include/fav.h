@@ -84,10 +84,14 @@ FAV_API fav_status fav_forward(const void *q, const void *k, const void *v, void
 /*
  * fav_forward_host -- the same operation on HOST buffers (end-to-end call).
  *
- * Copies q, k, v (host, ideally pinned) to internal device buffers, runs fav_forward on
- * `stream`, copies o and lse (lse may be NULL) back to the host and synchronises `stream`.
- * The device buffers grow on demand and are kept until fav_release_workspace().
- * Host pointers need no alignment.  Same argument rules and statuses as fav_forward.
+ * Copies q, k, v (host, ideally pinned) to internal device buffers, computes, copies o and lse
+ * (lse may be NULL) back to the host, and returns when the results are on the host.  The work
+ * is pipelined over up to four chunks of KV heads (batch and heads flattened), each chunk
+ * copied in, computed and copied out on three internal streams, so that copies in both
+ * directions overlap each other and the kernels.  It starts after the work already queued on
+ * `stream` (a cudaStream_t, NULL = legacy default stream).  The device buffers grow on demand
+ * and are kept until fav_release_workspace().  Host pointers need no alignment.  Same argument
+ * rules and statuses as fav_forward.
  */
 FAV_API fav_status fav_forward_host(const void *q, const void *k, const void *v, void *o, float *lse,
                             int B, int Hq, int Hkv, int Nq, int Nkv, int D,

@@ -29,7 +29,12 @@ struct DeviceState {
     size_t ws_bytes = 0;
     void *hbuf = nullptr;      // device copies for fav_forward_host
     size_t hbuf_bytes = 0;
+    bool pipe_init = false;    // fav_forward_host pipeline: copy-in, compute, copy-out streams
+    cudaStream_t s_in = nullptr, s_comp = nullptr, s_out = nullptr;
+    cudaEvent_t ev_start = nullptr, ev_in[4] = {}, ev_comp[4] = {};
 };
+
+constexpr int kHostChunks = 4;
 
 std::mutex g_mu;
 DeviceState g_dev[kMaxDevices];
@@ -252,24 +257,67 @@ fav_status fav_forward_host(const void *q, const void *k, const void *v, void *o
     uint8_t *base = nullptr;
     {
         std::lock_guard<std::mutex> lk(g_mu);
-        st = ensure_buffer(&ds->hbuf, &ds->hbuf_bytes, need, s);
+        if (!ds->pipe_init) {
+            bool okp = cudaStreamCreateWithFlags(&ds->s_in, cudaStreamNonBlocking) == cudaSuccess &&
+                       cudaStreamCreateWithFlags(&ds->s_comp, cudaStreamNonBlocking) == cudaSuccess &&
+                       cudaStreamCreateWithFlags(&ds->s_out, cudaStreamNonBlocking) == cudaSuccess &&
+                       cudaEventCreateWithFlags(&ds->ev_start, cudaEventDisableTiming) == cudaSuccess;
+            for (int c = 0; okp && c < kHostChunks; ++c)
+                okp = cudaEventCreateWithFlags(&ds->ev_in[c], cudaEventDisableTiming) == cudaSuccess &&
+                      cudaEventCreateWithFlags(&ds->ev_comp[c], cudaEventDisableTiming) == cudaSuccess;
+            if (!okp) return FAV_ERR_CUDA;
+            ds->pipe_init = true;
+        }
+        st = ensure_buffer(&ds->hbuf, &ds->hbuf_bytes, need, ds->s_comp);
         base = static_cast<uint8_t *>(ds->hbuf);
     }
     if (st != FAV_OK) return st;
     uint8_t *dq = base, *dk = dq + up(qb), *dv = dk + up(kb), *dout = dv + up(kb);
     float *dl = reinterpret_cast<float *>(dout + up(qb));
-    if (cudaMemcpyAsync(dq, q, qb, cudaMemcpyHostToDevice, s) != cudaSuccess ||
-        cudaMemcpyAsync(dk, k, kb, cudaMemcpyHostToDevice, s) != cudaSuccess ||
-        cudaMemcpyAsync(dv, v, kb, cudaMemcpyHostToDevice, s) != cudaSuccess)
+    // Pipeline over chunks of KV heads (batch and heads flattened: query head b*Hq + h reads KV
+    // head (b*Hq + h) / G = b*Hkv + h/G, so a chunk of KV heads owns a contiguous block of q, k,
+    // v, o and lse).  Chunk c is copied in on s_in, computed on s_comp, copied out on s_out;
+    // the three streams overlap across chunks.
+    const int G = Hq / Hkv;
+    const long long heads_kv = (long long)B * Hkv;
+    const int nch = (int)std::min<long long>(kHostChunks, heads_kv);
+    const size_t q_head = (size_t)Nq * D * es, kv_head = (size_t)Nkv * D * es, l_head = (size_t)Nq * 4;
+    const uint8_t *hq = static_cast<const uint8_t *>(q), *hk = static_cast<const uint8_t *>(k);
+    const uint8_t *hv = static_cast<const uint8_t *>(v);
+    uint8_t *ho = static_cast<uint8_t *>(o);
+    uint8_t *hl = reinterpret_cast<uint8_t *>(lse);
+    if (cudaEventRecord(ds->ev_start, s) != cudaSuccess ||
+        cudaStreamWaitEvent(ds->s_in, ds->ev_start, 0) != cudaSuccess ||
+        cudaStreamWaitEvent(ds->s_comp, ds->ev_start, 0) != cudaSuccess ||
+        cudaStreamWaitEvent(ds->s_out, ds->ev_start, 0) != cudaSuccess)
         return FAV_ERR_CUDA;
-    const FavArgs a = make_args(dq, dk, dv, dout, lse ? dl : nullptr, B, Hq, Hkv, Nq, Nkv, D,
-                                scale, causal, dtype);
-    st = forward_impl(a, s);
-    if (st != FAV_OK) return st;
-    if (cudaMemcpyAsync(o, dout, qb, cudaMemcpyDeviceToHost, s) != cudaSuccess) return FAV_ERR_CUDA;
-    if (lse && cudaMemcpyAsync(lse, dl, lb, cudaMemcpyDeviceToHost, s) != cudaSuccess)
-        return FAV_ERR_CUDA;
-    if (cudaStreamSynchronize(s) != cudaSuccess) return FAV_ERR_CUDA;
+    for (int c = 0; c < nch; ++c) {
+        const long long k0 = heads_kv * c / nch, k1 = heads_kv * (c + 1) / nch;
+        const size_t qo = (size_t)k0 * G * q_head, qn = (size_t)(k1 - k0) * G * q_head;
+        const size_t ko = (size_t)k0 * kv_head, kn = (size_t)(k1 - k0) * kv_head;
+        const size_t lo = (size_t)k0 * G * l_head, ln = (size_t)(k1 - k0) * G * l_head;
+        if (cudaMemcpyAsync(dq + qo, hq + qo, qn, cudaMemcpyHostToDevice, ds->s_in) != cudaSuccess ||
+            cudaMemcpyAsync(dk + ko, hk + ko, kn, cudaMemcpyHostToDevice, ds->s_in) != cudaSuccess ||
+            cudaMemcpyAsync(dv + ko, hv + ko, kn, cudaMemcpyHostToDevice, ds->s_in) != cudaSuccess ||
+            cudaEventRecord(ds->ev_in[c], ds->s_in) != cudaSuccess ||
+            cudaStreamWaitEvent(ds->s_comp, ds->ev_in[c], 0) != cudaSuccess)
+            return FAV_ERR_CUDA;
+        const FavArgs a = make_args(dq + qo, dk + ko, dv + ko, dout + qo,
+                                    lse ? dl + (size_t)k0 * G * Nq : nullptr, 1,
+                                    (int)((k1 - k0) * G), (int)(k1 - k0), Nq, Nkv, D, scale,
+                                    causal, dtype);
+        st = forward_impl(a, ds->s_comp);
+        if (st != FAV_OK) return st;
+        if (cudaEventRecord(ds->ev_comp[c], ds->s_comp) != cudaSuccess ||
+            cudaStreamWaitEvent(ds->s_out, ds->ev_comp[c], 0) != cudaSuccess ||
+            cudaMemcpyAsync(ho + qo, dout + qo, qn, cudaMemcpyDeviceToHost, ds->s_out) != cudaSuccess)
+            return FAV_ERR_CUDA;
+        if (lse && cudaMemcpyAsync(hl + lo, reinterpret_cast<uint8_t *>(dl) + lo, ln,
+                                   cudaMemcpyDeviceToHost, ds->s_out) != cudaSuccess)
+            return FAV_ERR_CUDA;
+    }
+    if (cudaStreamSynchronize(ds->s_out) != cudaSuccess) return FAV_ERR_CUDA;
+    if (cudaStreamSynchronize(ds->s_comp) != cudaSuccess) return FAV_ERR_CUDA;
     return FAV_OK;
 }
 

@@ -4,7 +4,7 @@ import pytest
 
 import paper_2608_18656_gb300 as fav
 from paper_2608_18656_gb300 import inputs as I
-from gpu_util import check, run_gpu, sample_rows
+from gpu_util import LSE_TOL, O_TOL, check, run_gpu, sample_rows
 
 pytestmark = pytest.mark.gpu
 
@@ -182,3 +182,31 @@ def test_prefill_head_pairings(Hq, Hkv):
     x = I.make_inputs(w)
     o, lse = run_gpu(w, x)
     check(w, o, lse, x)
+
+
+# ---- end-to-end host-buffer entry point ----
+
+@pytest.mark.parametrize("shape", [(I.F16, 1, 8, 8, 700, 700, 128, True),
+                                   (I.BF16, 2, 8, 2, 1, 3000, 128, False),
+                                   (I.BF16, 1, 6, 3, 333, 333, 64, False),
+                                   (I.F32, 1, 2, 2, 64, 64, 64, False)])
+def test_forward_host_matches_device(shape):
+    """fav_forward_host (pipelined over KV-head chunks) equals fav_forward: bit for bit on the
+    prefill and CUDA-core paths (the per-head arithmetic is the same); within the parity
+    tolerances on the decode path (a chunk may get a different split count)."""
+    import torch
+    dt, B, Hq, Hkv, Nq, Nkv, D, causal = shape
+    w = W(dt, B, Hq, Hkv, Nq, Nkv, D, causal=causal, seed=Nq + Hq)
+    x = I.make_inputs(w)
+    o_dev, lse_dev = run_gpu(w, x)
+    bits = {n: np.ascontiguousarray(x[n + "_bits"]) for n in ("q", "k", "v")}
+    o_host = np.empty_like(bits["q"])
+    lse_host = np.empty((B, Hq, Nq), np.float32)
+    fav.forward_host(bits["q"], bits["k"], bits["v"], o_host, lse_host, B, Hq, Hkv, Nq, Nkv, D,
+                     w.scale, causal, dt)
+    if Nq * (Hq // Hkv) <= 16 and dt != I.F32:
+        np.testing.assert_allclose(I.from_storage(o_host, dt), o_dev, rtol=0, atol=O_TOL[dt])
+        np.testing.assert_allclose(lse_host.astype(np.float64), lse_dev, rtol=0, atol=LSE_TOL)
+    else:
+        np.testing.assert_array_equal(I.from_storage(o_host, dt), o_dev)
+        np.testing.assert_array_equal(lse_host.astype(np.float64), lse_dev)
