@@ -53,12 +53,15 @@ class Dist:
         self.rank = int(os.environ.get("RANK", "0"))
         self.local = int(os.environ.get("LOCAL_RANK", "0"))
         self.pg = None
+        self.device = "cuda"
 
     def init(self, backend):
+        """One process group over the replicas (nccl on GPUs; gloo reduces on the CPU)."""
         if self.world > 1:
             import torch.distributed as dist
             dist.init_process_group(backend)
             self.pg = dist
+            self.device = "cpu" if backend == "gloo" else "cuda"
 
     def barrier(self):
         if self.pg:
@@ -68,13 +71,19 @@ class Dist:
         if not self.pg:
             return x
         import torch
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        t = torch.tensor([x], dtype=torch.float64, device=self.device)
         self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
         return float(t.item())
 
     def close(self):
         if self.pg:
             self.pg.destroy_process_group()
+
+
+def job_rate(units_per_rank, seconds_max, world):
+    """Whole-job throughput: every rank processes the same units (replicas, weak scaling),
+    and the job takes as long as its slowest rank."""
+    return units_per_rank * world / seconds_max
 
 
 # ---------------------------------------------------------------- clocks during timing
@@ -177,6 +186,13 @@ def time_device(fn, steps, warmup, stream, dist):
     import torch
     flush = torch.ones(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
     sink = torch.empty((), dtype=torch.uint8, device="cuda")
+    # Untimed ramp: keep the GPU busy for >= 0.2 s so that its clocks have left their idle
+    # state before the warm-up steps proper (a short timed run otherwise starts at idle clocks).
+    t_ramp = time.perf_counter()
+    while time.perf_counter() - t_ramp < 0.2:
+        for _ in range(20):
+            fn()
+        torch.cuda.synchronize()
     for _ in range(warmup):
         fn()
     torch.cuda.synchronize()
@@ -312,7 +328,7 @@ def fav_arm(args, dist):
             we = I.WORKLOADS[idx]
             _, mse, te, nle, pe = bench_workload(we, args.steps, args.warmup)
             if we.Nq == 1:
-                gbs = kv_bytes(we) / (mse * 1e-3) / 1e9 * dist.world
+                gbs = job_rate(kv_bytes(we), mse * 1e-3, dist.world) / 1e9
                 extras.append({"workload": we.name, "value": gbs, "unit": "GB/s",
                                "ms_per_step": mse, "path": pe, "kernel_launches_per_step": nle,
                                "roofline": {"bound": "hbm", "achieved": gbs / dist.world,
@@ -320,7 +336,7 @@ def fav_arm(args, dist):
                                             "frac": gbs / dist.world / pk["hbm_gbs"],
                                             "frac_of_nominal_7900": gbs / dist.world / 7900.0}})
             else:
-                tf = we.flops / (mse * 1e-3) / 1e12 * dist.world
+                tf = job_rate(we.flops, mse * 1e-3, dist.world) / 1e12
                 extras.append({"workload": we.name, "value": tf, "unit": "TFLOP/s",
                                "ms_per_step": mse, "path": pe, "kernel_launches_per_step": nle,
                                "roofline": {"bound": "tensor", "achieved": tf / dist.world,
@@ -328,13 +344,13 @@ def fav_arm(args, dist):
                                             "frac": tf / dist.world / pk["tflops"]}})
     clocks = sampler.stop() if sampler else None
 
-    value = w.flops * dist.world / (ms * 1e-3) / 1e12
+    value = job_rate(w.flops, ms * 1e-3, dist.world) / 1e12
     achieved = w.flops / (statistics.mean(times) * 1e-3) / 1e12
     e2e = None
     if True:
         e2e_s, h2d, d2h = time_e2e(fav, w, x, max(3, min(args.steps, 20)), 2)
         e2e_s = dist.max(e2e_s)
-        e2e = {"value": w.flops * dist.world / e2e_s / 1e12, "unit": "TFLOP/s",
+        e2e = {"value": job_rate(w.flops, e2e_s, dist.world) / 1e12, "unit": "TFLOP/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
     cpu = None
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu:

@@ -13,7 +13,8 @@
 //   * 128-key K and V tiles are streamed by TMA through a ring of shared-memory stages and
 //     serve both query tiles;
 //   * S_i = Q_i K^T (M = 128, N = 128, K = D) and O_i += P_i V (M = 128, N = D, K = 128) are
-//     tcgen05.mma issued by one thread, accumulating in tensor memory (TMEM).  P_i is written
+//     bursts of tcgen05.mma issued by one elected lane of a converged warp, accumulating in
+//     tensor memory (TMEM).  P_i is written
 //     back into TMEM over the columns of S_i and read from there by the P.V MMA;
 //   * one softmax warpgroup per query tile, one thread per query row (= TMEM lane): tcgen05.ld
 //     of its S row, mask, row max, exp2 in the log2 domain, row sum, P rounded to the I/O type,
@@ -27,11 +28,12 @@
 // when S_i(j) arrives: the softmax thread rescales it itself, before writing P_i(j).
 //
 // Warp roles (320 threads): warps 0-3 softmax of tile 0, warps 4-7 softmax of tile 1
-// (TMEM lane quarter = warp % 4); warp 8 = TMEM owner + MMA issuer (one thread); warp 9 = TMA
-// producer.  The issuing thread blocks while the tensor pipe is busy, and a wait on an
-// mbarrier costs it ~80 cycles of latency even when the phase is already complete; so it
-// tests the barriers it will need next *before* a burst of MMAs and looks at the answers
-// after it, and only waits for real on the ones that were not complete.
+// (TMEM lane quarter = warp % 4); warp 8 = TMEM owner + MMA issuer (the whole warp, one
+// elected lane issuing each burst); warp 9 = TMA producer.  The issuing lane blocks while the
+// tensor pipe is busy, and a wait on an mbarrier costs ~80 cycles of latency even when the
+// phase is already complete; so the warp tests the barriers it will need next *before* a
+// burst of MMAs and looks at the answers after it, and only waits for real on the ones that
+// were not complete.
 #include <cuda.h>
 #include <math.h>
 
@@ -234,105 +236,103 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             }
         }
     } else if (warp == kMmaWarp) {
-        // ---------------- MMA issuer ----------------
-        if (lane == 0) {
-            constexpr bool bf = IsBF16<T>::value;
-            constexpr uint32_t idesc_qk = fav::tc::idesc_f16(BM, BN, bf, false);
-            constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, bf, true);
-            // Descriptors are built once; a k-step only adds its byte offset (>> 4) to the
-            // start-address field, which cannot carry out of its 14 bits (addresses < 256 KB).
-            const uint64_t dq0 = fav::tc::sdesc_sw128(sbase + C::kOffQ, 16, 1024);
-            const uint64_t dk0 = fav::tc::sdesc_sw128(sK, 16, 1024);
-            const uint64_t dv0 = fav::tc::sdesc_sw128(sV, BN * 128, 1024);
-            // S_i = Q_i K_j^T
-            auto issue_s = [&](int i, int j) {
-                const uint64_t dq = dq0 + (uint64_t)((i * C::kQBytes) >> 4);
-                const uint64_t dk = dk0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4);
-                const uint32_t d_tmem = tmem + C::colS(i);
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint64_t koff = (uint64_t)((((kk >> 2) * (BM * 128)) + (kk & 3) * 32) >> 4);
-                    fav::tc::mma_ss(d_tmem, dq + koff, dk + koff, idesc_qk, kk > 0);
-                }
-            };
-            // O_i += P_i V_j, with P_i read from TMEM (8 columns = 16 keys per k-step; bf16 adds
-            // P_lo from 64 columns further) and V MN-major in shared memory (8-key groups
-            // 1024 B apart, 64-column blocks one box apart).
-            auto issue_pv = [&](int i, int j) {
-                const uint64_t dv = dv0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4);
-                const uint32_t s_tmem = tmem + C::colS(i);
-                const uint32_t o_tmem = tmem + C::colO(i);
-                const uint32_t acc = (j > 0) ? 1u : 0u;
-#pragma unroll
-                for (int kk = 0; kk < BN / 16; ++kk) {
-                    const uint64_t bd = dv + (uint64_t)((kk * 16 * 128) >> 4);
-                    fav::tc::mma_ts(o_tmem, s_tmem + kk * 8, bd, idesc_pv, acc | (kk > 0));
-                    if (kSplit) fav::tc::mma_ts(o_tmem, s_tmem + 64 + kk * 8, bd, idesc_pv, 1u);
-                }
-            };
+        // ---------------- MMA issuer: the whole warp, converged; one elected lane issues ----------------
+        constexpr bool bf = IsBF16<T>::value;
+        constexpr uint32_t idesc_qk = fav::tc::idesc_f16(BM, BN, bf, false);
+        constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, bf, true);
+        // Base descriptors are built once; a tile only adds its byte offset (>> 4) to the
+        // start-address field, which cannot carry out of its 14 bits (addresses < 256 KB).
+        const uint64_t dq0 = fav::tc::sdesc_sw128(sbase + C::kOffQ, 16, 1024);
+        const uint64_t dk0 = fav::tc::sdesc_sw128(sK, 16, 1024);
+        const uint64_t dv0 = fav::tc::sdesc_sw128(sV, BN * 128, 1024);
+        // S_i = Q_i K_j^T: D/16 k-steps over the 64-column boxes of Q_i and K_j.
+        auto issue_s = [&](int i, int j) {
+            fav::tc::mma_ss_burst_k128<D / 16>(
+                tmem + C::colS(i), dq0 + (uint64_t)((i * C::kQBytes) >> 4),
+                dk0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_qk, 0u);
+        };
+        // O_i += P_i V_j, with P_i read from TMEM (8 columns = 16 keys per k-step; bf16 adds
+        // P_lo from 64 columns further) and V MN-major in shared memory (8-key groups
+        // 1024 B apart, 64-column blocks one box apart).
+        auto issue_pv = [&](int i, int j) {
+            fav::tc::mma_ts_burst_k128<kSplit>(
+                tmem + C::colO(i), tmem + C::colS(i),
+                dv0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_pv, j > 0 ? 1u : 0u);
+        };
+        // Every lane waits; the outcome is made warp-uniform so that a bounded wait that gives
+        // up takes the whole warp out of the loop together (the bursts' elect.sync needs all
+        // 32 lanes).
+        auto wait_all = [&](uint32_t bar, uint32_t parity) {
+            return __all_sync(0xffffffffu, fav::mbar_wait(bar, parity, status));
+        };
+        auto wait_all_fast = [&](uint32_t bar, uint32_t parity) {
+            return __all_sync(0xffffffffu, fav::mbar_wait_fast(bar, parity, status));
+        };
+        auto try_all = [&](uint32_t bar, uint32_t parity) {
+            return __all_sync(0xffffffffu, fav::mbar_try(bar, parity));
+        };
 #ifdef FAV_TIMING
-            long long ts[16][6];
-            const long long t_start = t_ref;
+        long long ts[16][6];
+        const long long t_start = t_ref;
 #endif
-            bool ok = fav::mbar_wait(q_full, 0, status) && fav::mbar_wait(k_full, 0, status);
-            if (ok) {
-                fav::tc::fence_after();
+        bool ok = wait_all(q_full, 0) && wait_all(k_full, 0);
+        if (ok) {
+            fav::tc::fence_after();
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (n_kv_tiles[i] == 0) continue;
-                    issue_s(i, 0);
-                    fav::tc::commit(s_full + 8 * i);
-                }
-                fav::tc::commit(k_empty);
+            for (int i = 0; i < 2; ++i) {
+                if (n_kv_tiles[i] == 0) continue;
+                issue_s(i, 0);
+                fav::tc::commit_elect(s_full + 8 * i);
             }
-            // Issue order per key tile j: [P_0(j).V_j, S_0(j+1)], [P_1(j).V_j, S_1(j+1)]: the
-            // scores of the two tiles arrive half a period apart, so each softmax runs while the
-            // tensor core works on the other tile.
-            for (int j = 0; ok && j < n_kv; ++j) {
-                const int st = j % S, st1 = (j + 1) % S;
-                const bool nxt = j + 1 < n_kv;
-                // tested ahead: V_j now, K_{j+1} before the first burst, P_1(j) before the second
-                bool v_ready = fav::mbar_try(v_full + 8 * st, (j / S) & 1);
-                bool k_ready = !nxt;
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (j >= n_kv_tiles[i]) continue;
-                    FAV_STAMP(ts, j, 3 * i);
-                    if (!fav::mbar_wait_fast(p_full + 8 * i, j & 1, status)) { ok = false; break; }
-                    if (!v_ready) {
-                        if (!fav::mbar_wait(v_full + 8 * st, (j / S) & 1, status)) { ok = false; break; }
-                        v_ready = true;
-                    }
-                    FAV_STAMP(ts, j, 3 * i + 1);
-                    fav::tc::fence_after();
-                    const bool k_tested = k_ready || fav::mbar_try(k_full + 8 * st1, ((j + 1) / S) & 1);
-                    issue_pv(i, j);
-                    if (j + 1 < n_kv_tiles[i]) {
-                        if (!k_tested && !fav::mbar_wait(k_full + 8 * st1, ((j + 1) / S) & 1, status)) {
-                            ok = false;
-                            break;
-                        }
-                        k_ready = true;
-                        fav::tc::fence_after();
-                        issue_s(i, j + 1);
-                        fav::tc::commit(s_full + 8 * i);
-                    } else {
-                        fav::tc::commit(o_done + 8 * i);
-                    }
-                    FAV_STAMP(ts, j, 3 * i + 2);
-                }
-                if (!ok) break;
-                fav::tc::commit(v_empty + 8 * st);
-                if (nxt) fav::tc::commit(k_empty + 8 * st1);
-            }
-#ifdef FAV_TIMING
-            if (blockIdx.x == 0)
-                for (int j = 0; j < min(n_kv, 16); ++j)
-                    printf("[mma] j=%2d wait_p0 %6lld got_p0 %6lld done0 %6lld | wait_p1 %6lld got_p1 %6lld done1 %6lld\n", j,
-                           ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start, ts[j][3] - t_start,
-                           ts[j][4] - t_start, ts[j][5] - t_start);
-#endif
+            fav::tc::commit_elect(k_empty);
         }
+        // Issue order per key tile j: [P_0(j).V_j, S_0(j+1)], [P_1(j).V_j, S_1(j+1)]: the
+        // scores of the two tiles arrive half a period apart, so each softmax runs while the
+        // tensor core works on the other tile.
+        for (int j = 0; ok && j < n_kv; ++j) {
+            const int st = j % S, st1 = (j + 1) % S;
+            const bool nxt = j + 1 < n_kv;
+            // tested ahead: V_j now, K_{j+1} before the first burst
+            bool v_ready = try_all(v_full + 8 * st, (j / S) & 1);
+            bool k_ready = !nxt;
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                if (j >= n_kv_tiles[i]) continue;
+                FAV_STAMP(ts, j, 3 * i);
+                if (!wait_all_fast(p_full + 8 * i, j & 1)) { ok = false; break; }
+                if (!v_ready) {
+                    if (!wait_all(v_full + 8 * st, (j / S) & 1)) { ok = false; break; }
+                    v_ready = true;
+                }
+                FAV_STAMP(ts, j, 3 * i + 1);
+                fav::tc::fence_after();
+                const bool k_tested = k_ready || try_all(k_full + 8 * st1, ((j + 1) / S) & 1);
+                issue_pv(i, j);
+                if (j + 1 < n_kv_tiles[i]) {
+                    if (!k_tested && !wait_all(k_full + 8 * st1, ((j + 1) / S) & 1)) {
+                        ok = false;
+                        break;
+                    }
+                    k_ready = true;
+                    fav::tc::fence_after();
+                    issue_s(i, j + 1);
+                    fav::tc::commit_elect(s_full + 8 * i);
+                } else {
+                    fav::tc::commit_elect(o_done + 8 * i);
+                }
+                FAV_STAMP(ts, j, 3 * i + 2);
+            }
+            if (!ok) break;
+            fav::tc::commit_elect(v_empty + 8 * st);
+            if (nxt) fav::tc::commit_elect(k_empty + 8 * st1);
+        }
+#ifdef FAV_TIMING
+        if (blockIdx.x == 0 && lane == 0)
+            for (int j = 0; j < min(n_kv, 16); ++j)
+                printf("[mma] j=%2d wait_p0 %6lld got_p0 %6lld done0 %6lld | wait_p1 %6lld got_p1 %6lld done1 %6lld\n", j,
+                       ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start, ts[j][3] - t_start,
+                       ts[j][4] - t_start, ts[j][5] - t_start);
+#endif
     } else {
         // ---------------- softmax / correction / epilogue: one thread per query row ----------------
         const int i = warp >> 2;                          // query tile of this warpgroup
