@@ -73,8 +73,12 @@ typedef enum {
  *
  * Decode-shaped calls (small Nq * Hq / Hkv) split the key range over thread blocks and merge
  * the partial results with a log-sum-exp combine (associativity of the online softmax); the
- * partials live in an internal device workspace that grows on demand (cudaMallocAsync on
- * `stream`) and is kept until fav_release_workspace().  FAV_ERR_NO_MEMORY if that fails.
+ * partials live in an internal device workspace.  bf16 prefill computes P.V with fp16 weights:
+ * V is first converted to fp16 in an internal workspace under a power-of-two scale per KV head
+ * (exact for every element within 2^-31 of its head's largest |v|; smaller ones err by less
+ * than 2^-39 of it) and O is scaled back.  Both workspaces grow on demand (cudaMallocAsync on
+ * `stream`) and are kept until fav_release_workspace(); FAV_ERR_NO_MEMORY if that fails.
+ * Calls on different streams of one device share them: serialise such calls.
  * Returns FAV_OK once the kernels are enqueued; it does not synchronise.
  */
 FAV_API fav_status fav_forward(const void *q, const void *k, const void *v, void *o, float *lse,

@@ -27,6 +27,8 @@ struct DeviceState {
     int num_sms = 0;
     void *ws = nullptr;        // split-KV partials
     size_t ws_bytes = 0;
+    void *ws_pre = nullptr;    // prefill workspace (bf16: fp16 copy of V and its scales)
+    size_t ws_pre_bytes = 0;
     void *hbuf = nullptr;      // device copies for fav_forward_host
     size_t hbuf_bytes = 0;
     bool pipe_init = false;    // fav_forward_host pipeline: copy-in, compute, copy-out streams
@@ -143,9 +145,17 @@ fav_status forward_impl(const FavArgs &in, cudaStream_t stream) {
     case FAV_PATH_SIMT:
         st = fav_launch_simt(a, stream);
         break;
-    case FAV_PATH_PREFILL:
-        st = fav_launch_prefill(a, stream);
+    case FAV_PATH_PREFILL: {
+        void *ws = nullptr;
+        const size_t need = fav_prefill_workspace_bytes(a);
+        if (need) {
+            std::lock_guard<std::mutex> lk(g_mu);
+            st = ensure_buffer(&ds->ws_pre, &ds->ws_pre_bytes, need, stream);
+            ws = ds->ws_pre;
+        }
+        if (st == FAV_OK) st = fav_launch_prefill(a, ws, stream);
         break;
+    }
     case FAV_PATH_DECODE: {
         const int n_tiles = fav_decode_num_tiles(a);
         int splits = g_splits.load();
@@ -351,9 +361,10 @@ void fav_release_workspace(void) {
     DeviceState &d = g_dev[dev];
     cudaDeviceSynchronize();
     if (d.ws) cudaFree(d.ws);
+    if (d.ws_pre) cudaFree(d.ws_pre);
     if (d.hbuf) cudaFree(d.hbuf);
-    d.ws = d.hbuf = nullptr;
-    d.ws_bytes = d.hbuf_bytes = 0;
+    d.ws = d.ws_pre = d.hbuf = nullptr;
+    d.ws_bytes = d.ws_pre_bytes = d.hbuf_bytes = 0;
 }
 
 fav_status fav_set_path(fav_path p) {

@@ -30,7 +30,10 @@ fav_status fav_launch_decode(const FavArgs &a, int splits, void *workspace, cuda
 
 // tcgen05 prefill kernel (fav_prefill.cu).
 bool fav_prefill_supported(const FavArgs &a);
-fav_status fav_launch_prefill(const FavArgs &a, cudaStream_t s);
+// Device workspace the prefill launch needs (0 for fp16; bf16: the fp16 copy of V and its
+// per-head scales), and the launch itself with that workspace.
+size_t fav_prefill_workspace_bytes(const FavArgs &a);
+fav_status fav_launch_prefill(const FavArgs &a, void *workspace, cudaStream_t s);
 
 // With FAV_DEBUG_SYNC=1 in the environment: synchronise `s` after a launch and report a
 // failure of kernel `what` on stderr.  Returns true if the kernel failed.  No-op otherwise.

@@ -37,6 +37,7 @@
 #include <cuda.h>
 #include <math.h>
 
+#include <algorithm>
 #include <type_traits>
 
 #include "fav_device.cuh"
@@ -59,7 +60,12 @@ constexpr int kThreads = 320;
 constexpr int kMmaWarp = 8, kLoadWarp = 9;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kRescaleThreshold = 8.0f;   // log2 units: rescale when max grows by > 2^8
+constexpr float kRescaleThreshold = 4.0f;   // log2 units: rescale when max grows by > 2^4
+// The weights are stored as p * 2^kPShift (exponent reference m - kPShift): with the lazy
+// threshold they stay below 2^(4 + kPShift) = 2^15, inside fp16's range, and weights down to
+// 2^-25 of the reference stay fp16 normals.  O / l is unchanged (l carries the same factor);
+// the LSE subtracts kPShift.
+constexpr float kPShift = 11.0f;
 
 // 2^x for a pair of weights with ex2 on the special-function unit.  (Computing a share of them
 // with a polynomial on the FMA pipe was measured slower on this GPU: the softmax is bound by
@@ -81,13 +87,14 @@ __device__ __forceinline__ void static_for(F &&f) {
 template <typename T> struct IsBF16 { static constexpr bool value = false; };
 template <> struct IsBF16<__nv_bfloat16> { static constexpr bool value = true; };
 
-// With bf16 I/O the weights P are split as P = P_hi + P_lo with P_hi = bf16(p) and
-// P_lo = bf16(p - P_hi), and O accumulates P_hi.V + P_lo.V (two MMAs per k-step): together
-// they carry about 16 significant bits of each weight.  With a single bf16 P (8 bits) the
-// weights' rounding alone can move O by up to 2^-9 of |v| when a few weights dominate (any
-// reference maximum, lazy or not, leaves most of them inexact), which with the bf16 rounding
-// of O itself does not fit a 3e-3 error budget.  fp16 keeps 11 bits and uses one MMA.
-template <typename T> struct SplitP { static constexpr bool value = IsBF16<T>::value; };
+// Precision of the weights P in the P.V MMA.  A single bf16 P (8 significant bits) can move O
+// by up to 2^-9 of |v| when a few weights dominate (any reference maximum, lazy or not, leaves
+// most of them inexact), which with the bf16 rounding of O itself does not fit a 3e-3 error
+// budget.  So P is fp16 (11 bits, one MMA per k-step) for both I/O types: for bf16 I/O, V is
+// converted to fp16 first (fav_v16_kernel).  With the weights stored as p * 2^kPShift, fp16
+// weights down to 2^-25 of the reference are normal numbers; smaller ones err by at most
+// 2^-36 of it, which stays below the tolerance even next to a value of V 2^25 times larger
+// than the others.
 
 template <int D> struct PrefillCfg {
     static constexpr int kStages = (D == 128) ? 2 : 3;      // K/V ring depth
@@ -102,22 +109,25 @@ template <int D> struct PrefillCfg {
     static constexpr int kNumBars = 1 + 4 * kStages + 2 + 2 + 2;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
     static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
-    // TMEM columns: S0 | S1 | O0 | O1.  P_i aliases S_i: P_hi in its first 64 columns,
-    // P_lo (bf16 only) in the next 64.
+    // TMEM columns: S0 | S1 | O0 | O1.  P_i (fp16) aliases the first 64 columns of S_i.
     static constexpr uint32_t kTmemCols = 512;
     static __host__ __device__ constexpr uint32_t colS(int i) { return i ? 128u : 0u; }
     static __host__ __device__ constexpr uint32_t colO(int i) { return 256u + (i ? D : 0); }
     static_assert(256 + 2 * D <= 512, "TMEM budget");
 };
 
-template <typename T, int D>
+// bf16 I/O (kV16): Q, K and O are bf16; V has been converted to fp16 (tmV, scaled per KV head
+// by v_scale^-1, a power of two) so that P.V runs with fp16 weights, and the epilogue multiplies
+// O back by v_scale.  fp16 I/O: tmV is V itself.
+template <typename T, int D, bool kV16>
 __global__ void __launch_bounds__(kThreads, 1)
 fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, T *__restrict__ o,
-                   float *__restrict__ lse, int B, int Hq, int Hkv, int Nq, int Nkv,
-                   int n_qtiles, int pair_heads, float scale_log2, int causal, int *status) {
+                   float *__restrict__ lse, const float *__restrict__ v_scale, int B, int Hq,
+                   int Hkv, int Nq, int Nkv, int n_qtiles, int pair_heads, float scale_log2,
+                   int causal, int *status) {
     using C = PrefillCfg<D>;
-    constexpr bool kSplit = SplitP<T>::value;
+    using TP = __half;    // type of the weights P and of V in shared memory (P.V MMA)
     constexpr int S = C::kStages;
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment in the shared window (the 128-byte swizzle atom of TMA and MMA)
@@ -157,6 +167,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         t[1] = 2 * pr + 1;
     }
     const int bkv = b * Hkv + h[0] / G;
+    const float vsc = kV16 ? v_scale[bkv] : 1.f;     // V = v_scale * (fp16 copy)
     const int off = Nkv - Nq;                                   // bottom-right causal offset
     int n_kv_tiles[2];
 #pragma unroll
@@ -239,7 +250,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         // ---------------- MMA issuer: the whole warp, converged; one elected lane issues ----------------
         constexpr bool bf = IsBF16<T>::value;
         constexpr uint32_t idesc_qk = fav::tc::idesc_f16(BM, BN, bf, false);
-        constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, bf, true);
+        constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, false, true);      // fp16 P, V
         // Base descriptors are built once; a tile only adds its byte offset (>> 4) to the
         // start-address field, which cannot carry out of its 14 bits (addresses < 256 KB).
         const uint64_t dq0 = fav::tc::sdesc_sw128(sbase + C::kOffQ, 16, 1024);
@@ -251,13 +262,12 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                 tmem + C::colS(i), dq0 + (uint64_t)((i * C::kQBytes) >> 4),
                 dk0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_qk, 0u);
         };
-        // O_i += P_i V_j, with P_i read from TMEM (8 columns = 16 keys per k-step; bf16 adds
-        // P_lo from 64 columns further) and V MN-major in shared memory (8-key groups
-        // 1024 B apart, 64-column blocks one box apart).
+        // O_i += P_i V_j, with P_i read from TMEM (8 columns = 16 keys per k-step) and V
+        // MN-major in shared memory (8-key groups 1024 B apart, 64-column blocks one box apart).
         auto issue_pv = [&](int i, int j) {
-            fav::tc::mma_ts_burst_k128<kSplit>(
-                tmem + C::colO(i), tmem + C::colS(i),
-                dv0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_pv, j > 0 ? 1u : 0u);
+            fav::tc::mma_ts_burst_k128(tmem + C::colO(i), tmem + C::colS(i),
+                                       dv0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_pv,
+                                       j > 0 ? 1u : 0u);
         };
         // Every lane waits; the outcome is made warp-uniform so that a bounded wait that gives
         // up takes the whole warp out of the loop together (the bursts' elect.sync needs all
@@ -390,50 +400,30 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                 return fav::fmax3(fav::fmax3(m8[0], m8[1], m8[2]), fav::fmax3(m8[3], m8[4], m8[5]),
                                   fmaxf(m8[6], m8[7]));
             };
-            // p = exp2(s * scale_log2 - mref) on pairs (one packed FMA, two ex2, one packed
-            // add): packed weights, their fp32 sum, and the raw row maximum of the same pass.
-            uint32_t pk[2][32];
+            // p = exp2(s * scale_log2 - mref) on pairs (one packed FMA, two ex2, one packed add),
+            // fp16 weights stored to TMEM half a row at a time (keys [64h, 64h + 64) over S
+            // columns [32h, 32h + 32), whose scores are already in registers); returns nothing,
+            // accumulates the fp32 sum in psum.
             float psum = 0.f;
-            auto exp_pass = [&](float mref) {
+            auto exp_store = [&](float mref) {
                 const float2 sc2 = make_float2(scale_log2, scale_log2);
                 const float2 nm2 = make_float2(-mref, -mref);
                 float2 l4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                static_for<0, BN / 2>([&](auto pc) {
-                    constexpr int c = 2 * decltype(pc)::value;
-                    const float2 x = fav::ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
-                    const float2 p = exp2_pair<c / 2>(x);
-                    l4[(c >> 1) & 3] = fav::fadd2(l4[(c >> 1) & 3], p);
-                    m4[(c >> 1) & 3] = fav::fmax3(m4[(c >> 1) & 3], s[c], s[c + 1]);
-                    pk[c >> 6][(c >> 1) & 31] = fav::Elem<T>::pack(p.x, p.y);
+                static_for<0, 2>([&](auto hc) {
+                    constexpr int h = decltype(hc)::value;
+                    uint32_t pk[32];
+                    static_for<0, 32>([&](auto pc) {
+                        constexpr int e = 2 * decltype(pc)::value;
+                        constexpr int c = 64 * h + e;
+                        const float2 x = fav::ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
+                        const float2 p = exp2_pair<c / 2>(x);
+                        l4[(e >> 1) & 3] = fav::fadd2(l4[(e >> 1) & 3], p);
+                        pk[e >> 1] = fav::Elem<TP>::pack(p.x, p.y);
+                    });
+                    fav::tc::st_32x32b_x32(trow + colS + 32 * h, pk);
                 });
                 const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
                 psum = a.x + a.y;
-                return fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
-            };
-            // bf16: exponentials of keys [64h, 64h + 64) into hi / lo parts, stored to TMEM at
-            // once (P_hi over S columns [32h, 32h + 32), P_lo over [64 + 32h, 96 + 32h)).
-            auto exp_half_store = [&](float mref, int h) {
-                const float2 sc2 = make_float2(scale_log2, scale_log2);
-                const float2 nm2 = make_float2(-mref, -mref);
-                float2 l4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-                uint32_t hi32[32], lo32[32];
-                static_for<0, 32>([&](auto pe) {
-                    constexpr int e = 2 * decltype(pe)::value;
-                    const int c = 64 * h + e;
-                    const float2 x = fav::ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
-                    const float2 p = exp2_pair<e / 2>(x);
-                    l4[(e >> 1) & 3] = fav::fadd2(l4[(e >> 1) & 3], p);
-                    const uint32_t hi = fav::Elem<T>::pack(p.x, p.y);
-                    const float2 hf = make_float2(__uint_as_float(hi << 16), __uint_as_float(hi & 0xFFFF0000u));
-                    const float2 lo = fav::ffma2(hf, make_float2(-1.f, -1.f), p);
-                    hi32[e >> 1] = hi;
-                    lo32[e >> 1] = fav::Elem<T>::pack(lo.x, lo.y);
-                });
-                fav::tc::st_32x32b_x32(trow + colS + 32 * h, hi32);
-                fav::tc::st_32x32b_x32(trow + colS + 64 + 32 * h, lo32);
-                const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
-                psum += a.x + a.y;
             };
             float alpha = 1.f;
             bool rescale = false;
@@ -446,39 +436,15 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     l *= alpha;
                 }
             };
-            if constexpr (kSplit) {
-                // two passes: the row maximum first, then the weights, stored as produced
-                load_s();
-                FAV_STAMP(ts, j, 2);
-                move_max(row_max() * scale_log2);
-                FAV_STAMP(ts, j, 3);
-                psum = 0.f;
-                exp_half_store(m, 0);
-                exp_half_store(m, 1);
-            } else if (j == 0) {
-                load_s();
-                FAV_STAMP(ts, j, 2);
-                move_max(row_max() * scale_log2);
-                FAV_STAMP(ts, j, 3);
-                exp_pass(m);
-            } else {
-                // After the first tile the weights are computed speculatively against the
-                // current reference maximum while the tile's own maximum is found in the same
-                // pass; a warp with a row whose maximum grew by more than 2^8 (rare) reloads
-                // the scores and redoes the tile (warp-uniform: tcgen05.ld is collective).
-                load_s();
-                FAV_STAMP(ts, j, 2);
-                const bool redo = exp_pass(m) * scale_log2 > m + kRescaleThreshold;
-                FAV_STAMP(ts, j, 3);
-                if (__any_sync(~0u, redo)) {
-                    load_s();
-                    move_max(row_max() * scale_log2);
-                    exp_pass(m);
-                }
-            }
+            // two passes: the row maximum, then the weights against the (lazy) reference
+            load_s();
+            FAV_STAMP(ts, j, 2);
+            move_max(row_max() * scale_log2);
+            FAV_STAMP(ts, j, 3);
+            // P_i over the first 64 columns of S_i (two 16-bit weights per column)
+            exp_store(m - kPShift);
             l += psum;
             FAV_STAMP(ts, j, 4);
-            // (after the exponentials, so that only the packed weights are live)
             // O_i is stable here: P_i(j-1).V completed before S_i(j) (in-order MMAs, one commit).
             if (__any_sync(~0u, rescale)) {
 #pragma unroll
@@ -496,12 +462,6 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     }
                     fav::tc::st_32x32b_x32(trow + col, v);
                 }
-            }
-            // P_i over the first 64 columns of S_i (two 16-bit weights per column); bf16 has
-            // stored its hi and lo parts already.
-            if constexpr (!kSplit) {
-                fav::tc::st_32x32b_x32(trow + colS, pk[0]);
-                fav::tc::st_32x32b_x32(trow + colS + 32, pk[1]);
             }
             fav::tc::wait_st();
             fav::tc::fence_before();
@@ -523,7 +483,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         // ---------------- epilogue: O / l, LSE ----------------
         if (ok && n_mine > 0 && fav::mbar_wait(o_done + 8 * i, 0, status)) {
             fav::tc::fence_after();
-            const float inv_l = 1.f / l;
+            const float inv_l = vsc / l;
             const bool valid = qi < Nq;
             T *orow = o + ((long long)(b * Hq + hi) * Nq + qi) * D;
 #pragma unroll
@@ -543,7 +503,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     }
                 }
             }
-            if (valid && lse) lse[(long long)(b * Hq + hi) * Nq + qi] = (m + log2f(l)) * kLn2;
+            if (valid && lse) lse[(long long)(b * Hq + hi) * Nq + qi] = (m - kPShift + log2f(l)) * kLn2;
         }
     }
 
@@ -553,15 +513,116 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     if (warp == kMmaWarp) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
 }
 
-template <typename T, int D>
-fav_status launch(const FavArgs &a, cudaStream_t stream) {
+// ---- bf16 V -> fp16 V (per-KV-head power-of-two scale), for the kV16 kernel ----
+// Pass 1: per KV head, the largest finite |v| (as float bits: non-negative floats order like
+// their bit patterns, so an unsigned atomicMax finds it).
+__global__ void __launch_bounds__(256)
+fav_vmax_kernel(const uint4 *__restrict__ v, unsigned *__restrict__ vmax_bits, long long per_head) {
+    const long long head = blockIdx.y;
+    const uint4 *src = v + head * per_head;
+    unsigned mx = 0;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_head;
+         i += (long long)gridDim.x * blockDim.x) {
+        const uint4 w = src[i];
+        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            // two bf16 values: |x| bits are the low 15 bits of each half, moved to float bits
+            const uint32_t lo = (u[k] & 0x7FFFu) << 16, hi = u[k] & 0x7FFF0000u;
+            if (lo < 0x7F800000u) mx = max(mx, lo);      // finite only
+            if (hi < 0x7F800000u) mx = max(mx, hi);
+        }
+    }
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) mx = max(mx, __shfl_xor_sync(~0u, mx, d));
+    if ((threadIdx.x & 31) == 0 && mx) atomicMax(vmax_bits + head, mx);
+}
+
+// Scale exponent of a head: e = floor(log2(max|v|)) - 14, so that max|v| * 2^-e < 2^15 (fp16
+// max 65504); a head of zeros keeps e = 0.  Clamped to [-126, 127] so that 2^e and 2^-e are
+// both finite normal floats (a head whose maximum is below 2^-112 is scaled by 2^126 only).
+__device__ __forceinline__ int fav_v16_exponent(unsigned vmax_bits) {
+    if (vmax_bits == 0) return 0;
+    const int e2 = (int)(vmax_bits >> 23) - 127;        // floor(log2), -127 for subnormals
+    return min(127, max(-126, e2 - 14));
+}
+
+// Pass 2: v16 = fp16(v * 2^-e).  A bf16 value has 8 significant bits, which fp16 holds exactly
+// down to 2^-17 (subnormals included), so every |v| >= 2^(e-17) -- everything within about
+// 2^-31 of the head's maximum -- converts exactly; smaller values err by less than 2^(e-25).
+// Non-finite values stay non-finite.  Also stores v_scale = 2^e.
+__global__ void __launch_bounds__(256)
+fav_v16_kernel(const uint4 *__restrict__ v, uint4 *__restrict__ v16,
+               const unsigned *__restrict__ vmax_bits, float *__restrict__ v_scale,
+               long long per_head) {
+    const long long head = blockIdx.y;
+    const int e = fav_v16_exponent(vmax_bits[head]);
+    if (blockIdx.x == 0 && threadIdx.x == 0) v_scale[head] = ldexpf(1.f, e);
+    const float inv = ldexpf(1.f, -e);
+    const uint4 *src = v + head * per_head;
+    uint4 *dst = v16 + head * per_head;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_head;
+         i += (long long)gridDim.x * blockDim.x) {
+        const uint4 w = src[i];
+        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+        uint32_t r[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float lo = __uint_as_float(u[k] << 16) * inv;
+            const float hi = __uint_as_float(u[k] & 0xFFFF0000u) * inv;
+            r[k] = fav::Elem<__half>::pack(lo, hi);
+        }
+        dst[i] = make_uint4(r[0], r[1], r[2], r[3]);
+    }
+}
+
+// workspace of the kV16 path: [fp16 V][vmax bits per KV head][scale per KV head]
+struct V16Layout {
+    size_t v16, vmax, scale, total;
+    explicit V16Layout(const FavArgs &a) {
+        const size_t heads = (size_t)a.B * a.Hkv;
+        auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
+        v16 = 0;
+        vmax = up(heads * a.Nkv * a.D * 2);
+        scale = vmax + up(heads * 4);
+        total = scale + up(heads * 4);
+    }
+};
+
+template <typename T, int D, bool kV16>
+fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
     using C = PrefillCfg<D>;
+    const void *vsrc = a.v;
+    const float *v_scale = nullptr;
+    if constexpr (kV16) {
+        if (!workspace) return FAV_ERR_NO_MEMORY;
+        const V16Layout L(a);
+        uint8_t *ws = static_cast<uint8_t *>(workspace);
+        unsigned *vmax = reinterpret_cast<unsigned *>(ws + L.vmax);
+        float *vsc = reinterpret_cast<float *>(ws + L.scale);
+        const long long heads = (long long)a.B * a.Hkv;
+        const long long per_head = (long long)a.Nkv * a.D / 8;      // uint4 chunks (D % 8 == 0)
+        if (heads > 65535) return FAV_ERR_UNSUPPORTED;
+        const unsigned bx = (unsigned)std::max<long long>(
+            1, std::min<long long>((per_head + 255) / 256, std::max<long long>(1, 4LL * a.num_sms / heads)));
+        if (cudaMemsetAsync(vmax, 0, heads * sizeof(unsigned), stream) != cudaSuccess)
+            return FAV_ERR_CUDA;
+        fav_vmax_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(
+            static_cast<const uint4 *>(a.v), vmax, per_head);
+        fav_v16_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(
+            static_cast<const uint4 *>(a.v), reinterpret_cast<uint4 *>(ws + L.v16), vmax, vsc,
+            per_head);
+        if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_v16_kernel", stream))
+            return FAV_ERR_CUDA;
+        vsrc = ws + L.v16;
+        v_scale = vsc;
+    }
     alignas(64) CUtensorMap tmQ, tmK, tmV;
     fav_status st = fav_make_tmap_3d(&tmQ, a.q, D, a.Nq, a.B * a.Hq, BM);
     if (st == FAV_OK) st = fav_make_tmap_3d(&tmK, a.k, D, a.Nkv, a.B * a.Hkv, BN);
-    if (st == FAV_OK) st = fav_make_tmap_3d(&tmV, a.v, D, a.Nkv, a.B * a.Hkv, BN);
+    if (st == FAV_OK) st = fav_make_tmap_3d(&tmV, vsrc, D, a.Nkv, a.B * a.Hkv, BN);
     if (st != FAV_OK) return st;
-    auto kern = fav_prefill_kernel<T, D>;
+    auto kern = fav_prefill_kernel<T, D, kV16>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
         cudaSuccess)
         return FAV_ERR_CUDA;
@@ -572,8 +633,8 @@ fav_status launch(const FavArgs &a, cudaStream_t stream) {
                                         : (long long)((n_qtiles + 1) / 2) * a.B * a.Hq;
     if (blocks > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
     kern<<<(unsigned)blocks, kThreads, C::kSmemBytes, stream>>>(
-        tmQ, tmK, tmV, (T *)a.o, a.lse, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles, pair_heads,
-        a.scale * kLog2e, a.causal, a.dev_status);
+        tmQ, tmK, tmV, (T *)a.o, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
+        pair_heads, a.scale * kLog2e, a.causal, a.dev_status);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_kernel", stream))
         return FAV_ERR_CUDA;
     return FAV_OK;
@@ -587,8 +648,14 @@ bool fav_prefill_supported(const FavArgs &a) {
     return (long long)a.B * a.Hq <= 0x7fffffffLL && (long long)a.B * a.Hkv <= 0x7fffffffLL;
 }
 
-fav_status fav_launch_prefill(const FavArgs &a, cudaStream_t s) {
+size_t fav_prefill_workspace_bytes(const FavArgs &a) {
+    return a.dtype == FAV_BF16 ? V16Layout(a).total : 0;
+}
+
+fav_status fav_launch_prefill(const FavArgs &a, void *workspace, cudaStream_t s) {
     if (a.dtype == FAV_F16)
-        return a.D == 128 ? launch<__half, 128>(a, s) : launch<__half, 64>(a, s);
-    return a.D == 128 ? launch<__nv_bfloat16, 128>(a, s) : launch<__nv_bfloat16, 64>(a, s);
+        return a.D == 128 ? launch<__half, 128, false>(a, workspace, s)
+                          : launch<__half, 64, false>(a, workspace, s);
+    return a.D == 128 ? launch<__nv_bfloat16, 128, true>(a, workspace, s)
+                      : launch<__nv_bfloat16, 64, true>(a, workspace, s);
 }

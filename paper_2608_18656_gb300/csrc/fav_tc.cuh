@@ -128,37 +128,18 @@ __device__ __forceinline__ void mma_ss_burst_k128(uint32_t d_tmem, uint64_t ades
 
 // D (+)= A B over 8 k-steps of 16 (K = 128): A (M x 128 of 16-bit elements) read from TMEM,
 // 8 columns per k-step; B MN-major in shared memory, 16 rows of 128 bytes (2048 B) per k-step.
-// kSplit adds, per k-step, a second MMA with A taken 64 columns further (the low part of a
-// hi/lo split of A), accumulating onto the first.  `acc` = 0 overwrites D with the first MMA.
-template <bool kSplit>
+// `acc` = 0 overwrites D with the first MMA.
 __device__ __forceinline__ void mma_ts_burst_k128(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
                                                   uint32_t idesc, uint32_t acc) {
-    if constexpr (!kSplit) {
-        asm volatile(
-            "{\n\t.reg .pred e, p, t;\n\t.reg .b32 ta;\n\t.reg .b64 b1;\n\t"
-            "elect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\tsetp.eq.b32 t, %4, %4;\n\t"
-            "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
-            FAV_MMA_TS_STEP(8, 128) FAV_MMA_TS_STEP(16, 256) FAV_MMA_TS_STEP(24, 384)
-            FAV_MMA_TS_STEP(32, 512) FAV_MMA_TS_STEP(40, 640) FAV_MMA_TS_STEP(48, 768)
-            FAV_MMA_TS_STEP(56, 896)
-            "}"
-            ::"r"(d_tmem), "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(acc) : "memory");
-    } else {
-        asm volatile(
-            "{\n\t.reg .pred e, p, t;\n\t.reg .b32 ta;\n\t.reg .b64 b1;\n\t"
-            "elect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\tsetp.eq.b32 t, %4, %4;\n\t"
-            "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
-            FAV_MMA_TS_STEP(64, 0)
-            FAV_MMA_TS_STEP(8, 128) FAV_MMA_TS_STEP(72, 128)
-            FAV_MMA_TS_STEP(16, 256) FAV_MMA_TS_STEP(80, 256)
-            FAV_MMA_TS_STEP(24, 384) FAV_MMA_TS_STEP(88, 384)
-            FAV_MMA_TS_STEP(32, 512) FAV_MMA_TS_STEP(96, 512)
-            FAV_MMA_TS_STEP(40, 640) FAV_MMA_TS_STEP(104, 640)
-            FAV_MMA_TS_STEP(48, 768) FAV_MMA_TS_STEP(112, 768)
-            FAV_MMA_TS_STEP(56, 896) FAV_MMA_TS_STEP(120, 896)
-            "}"
-            ::"r"(d_tmem), "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(acc) : "memory");
-    }
+    asm volatile(
+        "{\n\t.reg .pred e, p, t;\n\t.reg .b32 ta;\n\t.reg .b64 b1;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\tsetp.eq.b32 t, %4, %4;\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
+        FAV_MMA_TS_STEP(8, 128) FAV_MMA_TS_STEP(16, 256) FAV_MMA_TS_STEP(24, 384)
+        FAV_MMA_TS_STEP(32, 512) FAV_MMA_TS_STEP(40, 640) FAV_MMA_TS_STEP(48, 768)
+        FAV_MMA_TS_STEP(56, 896)
+        "}"
+        ::"r"(d_tmem), "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(acc) : "memory");
 }
 #undef FAV_MMA_TS_STEP
 #undef FAV_MMA_TS_LO

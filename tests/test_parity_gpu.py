@@ -1,5 +1,7 @@
 """Parity of the CUDA path with the fp64 oracle on seeded inputs (needs a GB300)."""
 import numpy as np
+
+import oracle
 import pytest
 
 import paper_2608_18656_gb300 as fav
@@ -182,6 +184,36 @@ def test_prefill_head_pairings(Hq, Hkv):
     x = I.make_inputs(w)
     o, lse = run_gpu(w, x)
     check(w, o, lse, x)
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_prefill_bf16_v_range(D):
+    """bf16 prefill converts V to fp16 under a power-of-two scale per KV head: heads whose V
+    is far above or below fp16's range, a head of zeros, and a head with one large outlier
+    must all match the oracle.  Scaling the inputs by 2^k scales the exact output and every
+    rounding by 2^k, so the tolerance is the workloads' 3e-3 (which holds for |O| < 1) times
+    the power of two that brings the row's magnitude below 1."""
+    import torch
+    fav.set_path(fav.PATH_PREFILL)
+    w = W(I.BF16, 1, 10, 5, 300, 300, D, causal=True, seed=60 + D)
+    x = I.make_inputs(w)
+    v = x["v"].copy()
+    bulk = np.array([2.0 ** 20, 2.0 ** -40, 1000.0, 0.0, 1.0])
+    v *= bulk[None, :, None, None]
+    v[0, 4, 37, 5] = 2.0 ** 25                     # one outlier in an otherwise U(-1,1) head
+    v = I.round_to_dtype(v, I.BF16)
+    x = dict(x, v=v, v_bits=I.to_storage(v, I.BF16))
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_PREFILL
+    ro, rl = oracle.attention(x["q"], x["k"], x["v"], w.scale, w.causal)
+    assert np.isfinite(o).all()
+    G = w.Hq // w.Hkv
+    for h in range(w.Hq):
+        ref = ro[0, h]
+        mag = np.maximum(bulk[h // G], np.abs(ref).max(axis=1, keepdims=True))
+        tol = np.where(mag > 0, 3e-3 * np.exp2(np.ceil(np.log2(np.maximum(mag, 1e-300)))), 0.0)
+        assert (np.abs(o[0, h] - ref) <= tol).all(), "head %d" % h
+    assert np.abs(lse - rl).max() <= LSE_TOL
 
 
 # ---- end-to-end host-buffer entry point ----
