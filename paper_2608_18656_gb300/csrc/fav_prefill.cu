@@ -256,18 +256,19 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         const uint64_t dq0 = fav::tc::sdesc_sw128(sbase + C::kOffQ, 16, 1024);
         const uint64_t dk0 = fav::tc::sdesc_sw128(sK, 16, 1024);
         const uint64_t dv0 = fav::tc::sdesc_sw128(sV, BN * 128, 1024);
-        // S_i = Q_i K_j^T: D/16 k-steps over the 64-column boxes of Q_i and K_j.
-        auto issue_s = [&](int i, int j) {
+        // S_i = Q_i K_j^T: D/16 k-steps over the 64-column boxes of Q_i and K_j; the burst ends
+        // with commits to bar_a and bar_b (0 = none).
+        auto issue_s = [&](int i, int j, uint32_t bar_a, uint32_t bar_b) {
             fav::tc::mma_ss_burst_k128<D / 16>(
                 tmem + C::colS(i), dq0 + (uint64_t)((i * C::kQBytes) >> 4),
-                dk0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_qk, 0u);
+                dk0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_qk, 0u, bar_a, bar_b);
         };
         // O_i += P_i V_j, with P_i read from TMEM (8 columns = 16 keys per k-step) and V
         // MN-major in shared memory (8-key groups 1024 B apart, 64-column blocks one box apart).
-        auto issue_pv = [&](int i, int j) {
+        auto issue_pv = [&](int i, int j, uint32_t bar_a, uint32_t bar_b) {
             fav::tc::mma_ts_burst_k128(tmem + C::colO(i), tmem + C::colS(i),
                                        dv0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_pv,
-                                       j > 0 ? 1u : 0u);
+                                       j > 0 ? 1u : 0u, bar_a, bar_b);
         };
         // Every lane waits; the outcome is made warp-uniform so that a bounded wait that gives
         // up takes the whole warp out of the loop together (the bursts' elect.sync needs all
@@ -288,20 +289,21 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         bool ok = wait_all(q_full, 0) && wait_all(k_full, 0);
         if (ok) {
             fav::tc::fence_after();
+            const int last0 = n_kv_tiles[1] > 0 ? 1 : 0;      // last tile with work
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
                 if (n_kv_tiles[i] == 0) continue;
-                issue_s(i, 0);
-                fav::tc::commit_elect(s_full + 8 * i);
+                issue_s(i, 0, s_full + 8 * i, i == last0 ? k_empty : 0u);
             }
-            fav::tc::commit_elect(k_empty);
         }
         // Issue order per key tile j: [P_0(j).V_j, S_0(j+1)], [P_1(j).V_j, S_1(j+1)]: the
         // scores of the two tiles arrive half a period apart, so each softmax runs while the
-        // tensor core works on the other tile.
+        // tensor core works on the other tile.  The stage releases (v_empty, k_empty) are
+        // committed by the bursts of the last tile with work in this key tile.
         for (int j = 0; ok && j < n_kv; ++j) {
             const int st = j % S, st1 = (j + 1) % S;
             const bool nxt = j + 1 < n_kv;
+            const int last = j < n_kv_tiles[1] ? 1 : 0;
             // tested ahead: V_j now, K_{j+1} before the first burst
             bool v_ready = try_all(v_full + 8 * st, (j / S) & 1);
             bool k_ready = !nxt;
@@ -317,24 +319,21 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                 FAV_STAMP(ts, j, 3 * i + 1);
                 fav::tc::fence_after();
                 const bool k_tested = k_ready || try_all(k_full + 8 * st1, ((j + 1) / S) & 1);
-                issue_pv(i, j);
-                if (j + 1 < n_kv_tiles[i]) {
+                const bool more = j + 1 < n_kv_tiles[i];          // S_i(j+1) follows
+                issue_pv(i, j, i == last ? v_empty + 8 * st : 0u, more ? 0u : o_done + 8 * i);
+                if (more) {
                     if (!k_tested && !wait_all(k_full + 8 * st1, ((j + 1) / S) & 1)) {
                         ok = false;
                         break;
                     }
                     k_ready = true;
                     fav::tc::fence_after();
-                    issue_s(i, j + 1);
-                    fav::tc::commit_elect(s_full + 8 * i);
-                } else {
-                    fav::tc::commit_elect(o_done + 8 * i);
+                    issue_s(i, j + 1, s_full + 8 * i, i == last ? k_empty + 8 * st1 : 0u);
+                } else if (i == last && nxt) {
+                    fav::tc::commit_elect(k_empty + 8 * st1);   // another tile read K_{j+1}
                 }
                 FAV_STAMP(ts, j, 3 * i + 2);
             }
-            if (!ok) break;
-            fav::tc::commit_elect(v_empty + 8 * st);
-            if (nxt) fav::tc::commit_elect(k_empty + 8 * st1);
         }
 #ifdef FAV_TIMING
         if (blockIdx.x == 0 && lane == 0)

@@ -90,6 +90,13 @@ __device__ __forceinline__ void commit(uint32_t bar) {
 // MMA to be accepted, so every slot the other warps take from it between two MMAs idles the
 // tensor pipe).
 
+// After a burst, the issuing lane commits to barrier %5 and then %6 (shared-memory addresses;
+// 0 = no commit): each arrives once when every MMA this lane issued so far has completed.
+#define FAV_MMA_COMMITS                                                          \
+    "setp.ne.and.b32 ca, %5, 0, e;\n\tsetp.ne.and.b32 cb, %6, 0, e;\n\t"       \
+    "@ca tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%5];\n\t" \
+    "@cb tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%6];\n\t"
+
 #define FAV_MMA_SS_STEP(OFF)                                                     \
     "add.s64 a1, %1, " #OFF ";\n\tadd.s64 b1, %2, " #OFF ";\n\t"                 \
     "@e tcgen05.mma.cta_group::1.kind::f16 [%0], a1, b1, %3, t;\n\t"
@@ -99,25 +106,30 @@ __device__ __forceinline__ void commit(uint32_t bar) {
 // bytes into box kk / 4.  `acc` = 0 overwrites D with the first k-step.
 template <int NK>
 __device__ __forceinline__ void mma_ss_burst_k128(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                                  uint32_t idesc, uint32_t acc) {
+                                                  uint32_t idesc, uint32_t acc,
+                                                  uint32_t bar_a = 0, uint32_t bar_b = 0) {
     static_assert(NK == 4 || NK == 8, "k-steps per burst");
     if constexpr (NK == 4) {
         asm volatile(
-            "{\n\t.reg .pred e, p, t;\n\t.reg .b64 a1, b1;\n\t"
+            "{\n\t.reg .pred e, p, t, ca, cb;\n\t.reg .b64 a1, b1;\n\t"
             "elect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\tsetp.eq.b32 t, %4, %4;\n\t"
             "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t"
             FAV_MMA_SS_STEP(2) FAV_MMA_SS_STEP(4) FAV_MMA_SS_STEP(6)
+            FAV_MMA_COMMITS
             "}"
-            ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(acc) : "memory");
+            ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(acc), "r"(bar_a), "r"(bar_b)
+            : "memory");
     } else {
         asm volatile(
-            "{\n\t.reg .pred e, p, t;\n\t.reg .b64 a1, b1;\n\t"
+            "{\n\t.reg .pred e, p, t, ca, cb;\n\t.reg .b64 a1, b1;\n\t"
             "elect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\tsetp.eq.b32 t, %4, %4;\n\t"
             "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t"
             FAV_MMA_SS_STEP(2) FAV_MMA_SS_STEP(4) FAV_MMA_SS_STEP(6)
             FAV_MMA_SS_STEP(1024) FAV_MMA_SS_STEP(1026) FAV_MMA_SS_STEP(1028) FAV_MMA_SS_STEP(1030)
+            FAV_MMA_COMMITS
             "}"
-            ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(acc) : "memory");
+            ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(acc), "r"(bar_a), "r"(bar_b)
+            : "memory");
     }
 }
 #undef FAV_MMA_SS_STEP
@@ -130,19 +142,22 @@ __device__ __forceinline__ void mma_ss_burst_k128(uint32_t d_tmem, uint64_t ades
 // 8 columns per k-step; B MN-major in shared memory, 16 rows of 128 bytes (2048 B) per k-step.
 // `acc` = 0 overwrites D with the first MMA.
 __device__ __forceinline__ void mma_ts_burst_k128(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
-                                                  uint32_t idesc, uint32_t acc) {
+                                                  uint32_t idesc, uint32_t acc,
+                                                  uint32_t bar_a = 0, uint32_t bar_b = 0) {
     asm volatile(
-        "{\n\t.reg .pred e, p, t;\n\t.reg .b32 ta;\n\t.reg .b64 b1;\n\t"
+        "{\n\t.reg .pred e, p, t, ca, cb;\n\t.reg .b32 ta;\n\t.reg .b64 b1;\n\t"
         "elect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\tsetp.eq.b32 t, %4, %4;\n\t"
         "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
         FAV_MMA_TS_STEP(8, 128) FAV_MMA_TS_STEP(16, 256) FAV_MMA_TS_STEP(24, 384)
         FAV_MMA_TS_STEP(32, 512) FAV_MMA_TS_STEP(40, 640) FAV_MMA_TS_STEP(48, 768)
         FAV_MMA_TS_STEP(56, 896)
+        FAV_MMA_COMMITS
         "}"
-        ::"r"(d_tmem), "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(acc) : "memory");
+        ::"r"(d_tmem), "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(acc), "r"(bar_a), "r"(bar_b)
+        : "memory");
 }
 #undef FAV_MMA_TS_STEP
-#undef FAV_MMA_TS_LO
+#undef FAV_MMA_COMMITS
 
 // commit() from a converged warp: one elected lane commits.
 __device__ __forceinline__ void commit_elect(uint32_t bar) {
