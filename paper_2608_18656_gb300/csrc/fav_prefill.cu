@@ -311,7 +311,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             for (int i = 0; i < 2; ++i) {
                 if (j >= n_kv_tiles[i]) continue;
                 FAV_STAMP(ts, j, 3 * i);
-                if (!wait_all_fast(p_full + 8 * i, j & 1)) { ok = false; break; }
+                if (!wait_all(p_full + 8 * i, j & 1)) { ok = false; break; }
                 if (!v_ready) {
                     if (!wait_all(v_full + 8 * st, (j / S) & 1)) { ok = false; break; }
                     v_ready = true;
