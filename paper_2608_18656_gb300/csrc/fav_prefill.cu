@@ -106,7 +106,7 @@ template <int D> struct PrefillCfg {
     static constexpr int kOffK = kOffQ + 2 * kQBytes;
     static constexpr int kOffV = kOffK + kStages * kKVBytes;
     static constexpr int kOffBar = kOffV + kStages * kKVBytes;
-    static constexpr int kNumBars = 1 + 4 * kStages + 2 + 2 + 2;
+    static constexpr int kNumBars = 2 + 1 + 4 * kStages + 2 + 2 + 2;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
     static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
     // TMEM columns: S0 | S1 | O0 | O1.  P_i (fp16) aliases the first 64 columns of S_i.
@@ -136,8 +136,9 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     const uint32_t sbase = fav::smem_u32(smem);
     const uint32_t sK = sbase + C::kOffK, sV = sbase + C::kOffV;
     const uint32_t bar0 = sbase + C::kOffBar;
-    const uint32_t q_full = bar0;
-    const uint32_t k_full = bar0 + 8, k_empty = k_full + 8 * S;
+    const uint32_t q_full = bar0;                 // [2], one per query tile
+    const uint32_t q_empty = q_full + 16;         // Q buffers free (last S MMA of a unit done)
+    const uint32_t k_full = q_empty + 8, k_empty = k_full + 8 * S;
     const uint32_t v_full = k_empty + 8 * S, v_empty = v_full + 8 * S;
     const uint32_t s_full = v_empty + 8 * S;      // [2], one per query tile
     const uint32_t p_full = s_full + 16;          // [2]
@@ -146,45 +147,61 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int G = Hq / Hkv;
-
-    // ---- the two query tiles of this CTA (heaviest causal work first) ----
-    int b, h[2], t[2];
-    if (pair_heads) {
-        const int units = B * (Hq / 2);
-        const int u = blockIdx.x % units;
-        t[0] = t[1] = n_qtiles - 1 - (int)(blockIdx.x / units);
-        b = u / (Hq / 2);
-        h[0] = 2 * (u % (Hq / 2));
-        h[1] = h[0] + 1;
-    } else {
-        const int BH = B * Hq;
-        const int n_pairs = (n_qtiles + 1) / 2;
-        const int bh = blockIdx.x % BH;
-        const int pr = n_pairs - 1 - (int)(blockIdx.x / BH);
-        b = bh / Hq;
-        h[0] = h[1] = bh % Hq;
-        t[0] = 2 * pr;
-        t[1] = 2 * pr + 1;
-    }
-    const int bkv = b * Hkv + h[0] / G;
-    const float vsc = kV16 ? v_scale[bkv] : 1.f;     // V = v_scale * (fp16 copy)
     const int off = Nkv - Nq;                                   // bottom-right causal offset
-    int n_kv_tiles[2];
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-        if (t[i] >= n_qtiles) {
-            n_kv_tiles[i] = 0;
+
+    // ---- work units: two query tiles that read the same K/V head, heaviest causal first ----
+    // Unit u: the same query tile of two heads of one GQA group (even group sizes), or two
+    // consecutive query tiles of one head.  The CTA takes units c, 2P-1-c, 2P+c, 4P-1-c, ...
+    // (P CTAs, "snake" order): with the units sorted by decreasing work, this evens out the
+    // sums per CTA.
+    struct Unit {
+        int b, h[2], t[2], n_kv_tiles[2], n_kv, bkv;
+    };
+    const int n_units = pair_heads ? n_qtiles * B * (Hq / 2) : ((n_qtiles + 1) / 2) * B * Hq;
+    auto unit_at = [&](int k) {   // the k-th unit of this CTA, or -1
+        const int P = gridDim.x, c = blockIdx.x;
+        const int u = k * P + ((k & 1) ? (P - 1 - c) : c);
+        return u < n_units ? u : -1;
+    };
+    auto make_unit = [&](int u) {
+        Unit U;
+        if (pair_heads) {
+            const int units = B * (Hq / 2);
+            const int r = u % units;
+            U.t[0] = U.t[1] = n_qtiles - 1 - u / units;
+            U.b = r / (Hq / 2);
+            U.h[0] = 2 * (r % (Hq / 2));
+            U.h[1] = U.h[0] + 1;
         } else {
-            const int kv_end = causal ? min(Nkv, t[i] * BM + BM + off) : Nkv;
-            n_kv_tiles[i] = (kv_end + BN - 1) / BN;
+            const int BH = B * Hq;
+            const int n_pairs = (n_qtiles + 1) / 2;
+            const int bh = u % BH;
+            const int pr = n_pairs - 1 - u / BH;
+            U.b = bh / Hq;
+            U.h[0] = U.h[1] = bh % Hq;
+            U.t[0] = 2 * pr;
+            U.t[1] = 2 * pr + 1;
         }
-    }
-    const int n_kv = max(n_kv_tiles[0], n_kv_tiles[1]);
+        U.bkv = U.b * Hkv + U.h[0] / G;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            if (U.t[i] >= n_qtiles) {
+                U.n_kv_tiles[i] = 0;
+            } else {
+                const int kv_end = causal ? min(Nkv, U.t[i] * BM + BM + off) : Nkv;
+                U.n_kv_tiles[i] = (kv_end + BN - 1) / BN;
+            }
+        }
+        U.n_kv = max(U.n_kv_tiles[0], U.n_kv_tiles[1]);
+        return U;
+    };
 
     if (warp == kLoadWarp && lane == 0) {
         (void)FAV_CHECK((sbase & 1023u) == 0, status);
         (void)FAV_CHECK((sbase - raw_u32) + C::kOffTmemSlot + 4 <= fav::dynamic_smem_bytes(), status);
         fav::mbar_init(q_full, 1);
+        fav::mbar_init(q_full + 8, 1);
+        fav::mbar_init(q_empty, 1);
         for (int s = 0; s < S; ++s) {
             fav::mbar_init(k_full + 8 * s, 1);
             fav::mbar_init(k_empty + 8 * s, 1);
@@ -212,38 +229,47 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     const uint32_t tmem = *tmem_slot;
     (void)FAV_CHECK((tmem & 0xFFFFu) + C::kTmemCols <= 512u && (tmem >> 16) == 0u, status);
 
+    // Barrier phases run on across units: K/V stages follow one sequence g of key tiles
+    // (stage g % S, parity (g / S) & 1) on both sides; s_full / p_full of tile i complete once
+    // per key tile of i, o_done once per unit in which tile i has work, q_full once per unit.
     if (warp == kLoadWarp) {
         // ---------------- TMA producer ----------------
         if (lane == 0) {
             fav::tma_prefetch_desc(&tmQ);
             fav::tma_prefetch_desc(&tmK);
             fav::tma_prefetch_desc(&tmV);
-            const int nq = (n_kv_tiles[0] > 0) + (n_kv_tiles[1] > 0);
-            fav::mbar_arrive_expect_tx(q_full, nq * C::kQBytes);
+            int g = 0;
+            bool ok = true;
+            for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
+                const Unit U = make_unit(u);
+                // the Q buffers are free once the previous unit's last S MMA has completed; both
+                // tiles are loaded (a tile beyond the sequence reads the zero fill)
+                if (k > 0 && !fav::mbar_wait(q_empty, (k - 1) & 1, status)) break;
 #pragma unroll
-            for (int i = 0; i < 2; ++i) {
-                if (n_kv_tiles[i] == 0) continue;
+                for (int i = 0; i < 2; ++i) {
+                    fav::mbar_arrive_expect_tx(q_full + 8 * i, C::kQBytes);
 #pragma unroll
-                for (int bx = 0; bx < C::kBoxes; ++bx)
-                    fav::tma_load_3d(sbase + C::kOffQ + i * C::kQBytes + bx * BM * 128, &tmQ, q_full,
-                                     bx * 64, t[i] * BM, b * Hq + h[i]);
-            }
-            // Each stage has its own empty barriers (one commit per use, waited in order).
-            for (int j = 0; j < n_kv; ++j) {
-                const int st = j % S;
-                const uint32_t ph = ((j / S) + 1) & 1;   // parity of the previous use's phase
-                if (j >= S && !fav::mbar_wait(k_empty + 8 * st, ph, status)) break;
-                fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
+                    for (int bx = 0; bx < C::kBoxes; ++bx)
+                        fav::tma_load_3d(sbase + C::kOffQ + i * C::kQBytes + bx * BM * 128, &tmQ,
+                                         q_full + 8 * i, bx * 64, U.t[i] * BM, U.b * Hq + U.h[i]);
+                }
+                // Each stage has its own empty barriers (one commit per use, waited in order).
+                for (int j = 0; j < U.n_kv; ++j, ++g) {
+                    const int st = g % S;
+                    const uint32_t ph = ((g / S) + 1) & 1;   // parity of the previous use's phase
+                    if (g >= S && !fav::mbar_wait(k_empty + 8 * st, ph, status)) { ok = false; break; }
+                    fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
 #pragma unroll
-                for (int bx = 0; bx < C::kBoxes; ++bx)
-                    fav::tma_load_3d(sK + st * C::kKVBytes + bx * BN * 128, &tmK, k_full + 8 * st,
-                                     bx * 64, j * BN, bkv);
-                if (j >= S && !fav::mbar_wait(v_empty + 8 * st, ph, status)) break;
-                fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
+                    for (int bx = 0; bx < C::kBoxes; ++bx)
+                        fav::tma_load_3d(sK + st * C::kKVBytes + bx * BN * 128, &tmK, k_full + 8 * st,
+                                         bx * 64, j * BN, U.bkv);
+                    if (g >= S && !fav::mbar_wait(v_empty + 8 * st, ph, status)) { ok = false; break; }
+                    fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
 #pragma unroll
-                for (int bx = 0; bx < C::kBoxes; ++bx)
-                    fav::tma_load_3d(sV + st * C::kKVBytes + bx * BN * 128, &tmV, v_full + 8 * st,
-                                     bx * 64, j * BN, bkv);
+                    for (int bx = 0; bx < C::kBoxes; ++bx)
+                        fav::tma_load_3d(sV + st * C::kKVBytes + bx * BN * 128, &tmV, v_full + 8 * st,
+                                         bx * 64, j * BN, U.bkv);
+                }
             }
         }
     } else if (warp == kMmaWarp) {
@@ -256,28 +282,25 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         const uint64_t dq0 = fav::tc::sdesc_sw128(sbase + C::kOffQ, 16, 1024);
         const uint64_t dk0 = fav::tc::sdesc_sw128(sK, 16, 1024);
         const uint64_t dv0 = fav::tc::sdesc_sw128(sV, BN * 128, 1024);
-        // S_i = Q_i K_j^T: D/16 k-steps over the 64-column boxes of Q_i and K_j; the burst ends
-        // with commits to bar_a and bar_b (0 = none).
-        auto issue_s = [&](int i, int j, uint32_t bar_a, uint32_t bar_b) {
+        // S_i = Q_i K^T (K in ring stage st): D/16 k-steps over the 64-column boxes of Q_i and
+        // K; the burst ends with commits to bar_a and bar_b (0 = none).
+        auto issue_s = [&](int i, int st, uint32_t bar_a, uint32_t bar_b) {
             fav::tc::mma_ss_burst_k128<D / 16>(
                 tmem + C::colS(i), dq0 + (uint64_t)((i * C::kQBytes) >> 4),
-                dk0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_qk, 0u, bar_a, bar_b);
+                dk0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_qk, 0u, bar_a, bar_b);
         };
-        // O_i += P_i V_j, with P_i read from TMEM (8 columns = 16 keys per k-step) and V
-        // MN-major in shared memory (8-key groups 1024 B apart, 64-column blocks one box apart).
-        auto issue_pv = [&](int i, int j, uint32_t bar_a, uint32_t bar_b) {
+        // O_i (+)= P_i V, with P_i read from TMEM (8 columns = 16 keys per k-step) and V MN-major
+        // in shared memory (8-key groups 1024 B apart, 64-column blocks one box apart).
+        auto issue_pv = [&](int i, int st, uint32_t acc, uint32_t bar_a, uint32_t bar_b) {
             fav::tc::mma_ts_burst_k128(tmem + C::colO(i), tmem + C::colS(i),
-                                       dv0 + (uint64_t)(((j % S) * C::kKVBytes) >> 4), idesc_pv,
-                                       j > 0 ? 1u : 0u, bar_a, bar_b);
+                                       dv0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_pv, acc,
+                                       bar_a, bar_b);
         };
         // Every lane waits; the outcome is made warp-uniform so that a bounded wait that gives
         // up takes the whole warp out of the loop together (the bursts' elect.sync needs all
         // 32 lanes).
         auto wait_all = [&](uint32_t bar, uint32_t parity) {
             return __all_sync(0xffffffffu, fav::mbar_wait(bar, parity, status));
-        };
-        auto wait_all_fast = [&](uint32_t bar, uint32_t parity) {
-            return __all_sync(0xffffffffu, fav::mbar_wait_fast(bar, parity, status));
         };
         auto try_all = [&](uint32_t bar, uint32_t parity) {
             return __all_sync(0xffffffffu, fav::mbar_try(bar, parity));
@@ -286,205 +309,227 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         long long ts[16][6];
         const long long t_start = t_ref;
 #endif
-        bool ok = wait_all(q_full, 0) && wait_all(k_full, 0);
-        if (ok) {
+        int g = 0;                 // key tiles streamed so far (ring sequence)
+        int np[2] = {0, 0};        // P_i(.) consumed so far, per tile (p_full parity)
+        bool ok = true;
+        for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
+            const Unit U = make_unit(u);
+            const int g0 = g;
+            // first scores of the unit (the previous unit's last P.V are ahead in the pipe, so
+            // S_i(0) cannot overwrite its P_i before it is read)
+            const int last0 = U.n_kv_tiles[1] > 0 ? 1 : 0;      // last tile with work
+            ok = wait_all(q_full, k & 1) && wait_all(k_full + 8 * (g0 % S), (g0 / S) & 1);
+            if (!ok) break;
             fav::tc::fence_after();
-            const int last0 = n_kv_tiles[1] > 0 ? 1 : 0;      // last tile with work
-#pragma unroll
-            for (int i = 0; i < 2; ++i) {
-                if (n_kv_tiles[i] == 0) continue;
-                issue_s(i, 0, s_full + 8 * i, i == last0 ? k_empty : 0u);
-            }
-        }
-        // Issue order per key tile j: [P_0(j).V_j, S_0(j+1)], [P_1(j).V_j, S_1(j+1)]: the
-        // scores of the two tiles arrive half a period apart, so each softmax runs while the
-        // tensor core works on the other tile.  The stage releases (v_empty, k_empty) are
-        // committed by the bursts of the last tile with work in this key tile.
-        for (int j = 0; ok && j < n_kv; ++j) {
-            const int st = j % S, st1 = (j + 1) % S;
-            const bool nxt = j + 1 < n_kv;
-            const int last = j < n_kv_tiles[1] ? 1 : 0;
-            // tested ahead: V_j now, K_{j+1} before the first burst
-            bool v_ready = try_all(v_full + 8 * st, (j / S) & 1);
-            bool k_ready = !nxt;
-#pragma unroll
-            for (int i = 0; i < 2; ++i) {
-                if (j >= n_kv_tiles[i]) continue;
-                FAV_STAMP(ts, j, 3 * i);
-                if (!wait_all(p_full + 8 * i, j & 1)) { ok = false; break; }
-                if (!v_ready) {
-                    if (!wait_all(v_full + 8 * st, (j / S) & 1)) { ok = false; break; }
-                    v_ready = true;
-                }
-                FAV_STAMP(ts, j, 3 * i + 1);
+            issue_s(0, g0 % S, s_full, last0 == 0 ? k_empty + 8 * (g0 % S) : 0u);
+            if (last0 == 1) {
+                if (!(ok = wait_all(q_full + 8, k & 1))) break;
                 fav::tc::fence_after();
-                const bool k_tested = k_ready || try_all(k_full + 8 * st1, ((j + 1) / S) & 1);
-                const bool more = j + 1 < n_kv_tiles[i];          // S_i(j+1) follows
-                issue_pv(i, j, i == last ? v_empty + 8 * st : 0u, more ? 0u : o_done + 8 * i);
-                if (more) {
-                    if (!k_tested && !wait_all(k_full + 8 * st1, ((j + 1) / S) & 1)) {
-                        ok = false;
-                        break;
-                    }
-                    k_ready = true;
-                    fav::tc::fence_after();
-                    issue_s(i, j + 1, s_full + 8 * i, i == last ? k_empty + 8 * st1 : 0u);
-                } else if (i == last && nxt) {
-                    fav::tc::commit_elect(k_empty + 8 * st1);   // another tile read K_{j+1}
-                }
-                FAV_STAMP(ts, j, 3 * i + 2);
+                issue_s(1, g0 % S, s_full + 8, k_empty + 8 * (g0 % S));
             }
-        }
+            if (U.n_kv == 1) fav::tc::commit_elect(q_empty);    // no further S in this unit
+            // Issue order per key tile j: [P_0(j).V_j, S_0(j+1)], [P_1(j).V_j, S_1(j+1)]: the
+            // scores of the two tiles arrive half a period apart, so each softmax runs while the
+            // tensor core works on the other tile.  The stage releases (v_empty, k_empty) are
+            // committed by the bursts of the last tile with work in this key tile.
+            for (int j = 0; ok && j < U.n_kv; ++j) {
+                const int gj = g0 + j;
+                const int st = gj % S, st1 = (gj + 1) % S;
+                const bool nxt = j + 1 < U.n_kv;
+                const int last = j < U.n_kv_tiles[1] ? 1 : 0;
+                // tested ahead: V_j now, K_{j+1} before the first burst
+                bool v_ready = try_all(v_full + 8 * st, (gj / S) & 1);
+                bool k_ready = !nxt;
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (j >= U.n_kv_tiles[i]) continue;
+                    if (k == 0) FAV_STAMP(ts, j, 3 * i);
+                    if (!wait_all(p_full + 8 * i, np[i] & 1)) { ok = false; break; }
+                    ++np[i];
+                    if (!v_ready) {
+                        if (!wait_all(v_full + 8 * st, (gj / S) & 1)) { ok = false; break; }
+                        v_ready = true;
+                    }
+                    if (k == 0) FAV_STAMP(ts, j, 3 * i + 1);
+                    fav::tc::fence_after();
+                    const bool k_tested = k_ready || try_all(k_full + 8 * st1, ((gj + 1) / S) & 1);
+                    const bool more = j + 1 < U.n_kv_tiles[i];          // S_i(j+1) follows
+                    issue_pv(i, st, j > 0 ? 1u : 0u, i == last ? v_empty + 8 * st : 0u,
+                             more ? 0u : o_done + 8 * i);
+                    if (more) {
+                        if (!k_tested && !wait_all(k_full + 8 * st1, ((gj + 1) / S) & 1)) {
+                            ok = false;
+                            break;
+                        }
+                        k_ready = true;
+                        fav::tc::fence_after();
+                        issue_s(i, st1, s_full + 8 * i, i == last ? k_empty + 8 * st1 : 0u);
+                    } else if (i == last && nxt) {
+                        fav::tc::commit_elect(k_empty + 8 * st1);   // another tile read K_{j+1}
+                    }
+                    if (k == 0) FAV_STAMP(ts, j, 3 * i + 2);
+                }
+                // after the unit's last scores (issued in this key tile), its Q buffers can be
+                // refilled: the commit covers every MMA issued so far
+                if (ok && j + 2 == U.n_kv) fav::tc::commit_elect(q_empty);
+            }
+            g += U.n_kv;
 #ifdef FAV_TIMING
-        if (blockIdx.x == 0 && lane == 0)
-            for (int j = 0; j < min(n_kv, 16); ++j)
-                printf("[mma] j=%2d wait_p0 %6lld got_p0 %6lld done0 %6lld | wait_p1 %6lld got_p1 %6lld done1 %6lld\n", j,
-                       ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start, ts[j][3] - t_start,
-                       ts[j][4] - t_start, ts[j][5] - t_start);
+            if (k == 0 && blockIdx.x == 0 && lane == 0)
+                for (int j = 0; j < min(U.n_kv, 16); ++j)
+                    printf("[mma] j=%2d wait_p0 %6lld got_p0 %6lld done0 %6lld | wait_p1 %6lld got_p1 %6lld done1 %6lld\n", j,
+                           ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start, ts[j][3] - t_start,
+                           ts[j][4] - t_start, ts[j][5] - t_start);
 #endif
+        }
     } else {
         // ---------------- softmax / correction / epilogue: one thread per query row ----------------
         const int i = warp >> 2;                          // query tile of this warpgroup
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;
-        const int ti = i ? t[1] : t[0];
-        const int hi = i ? h[1] : h[0];
-        const int q0 = ti * BM;
-        const int qi = q0 + row;                          // query index of this row
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
         const uint32_t colS = i ? C::colS(1) : C::colS(0);
         const uint32_t colO = i ? C::colO(1) : C::colO(0);
-        const int lim = causal ? min(Nkv, qi + off + 1) : Nkv;       // visible keys: [0, lim)
-        const int lim_tile = causal ? min(Nkv, q0 + off + 1) : Nkv;  // smallest lim in the tile
-        const int n_mine = i ? n_kv_tiles[1] : n_kv_tiles[0];
-        float m = -INFINITY, l = 0.f;
+        int ns = 0, no = 0;        // S_i(.) and O_i completions consumed so far (parities)
         bool ok = true;
 #ifdef FAV_TIMING
         long long ts[16][6];
         const long long t_start = t_ref;
 #endif
-        for (int j = 0; j < n_mine; ++j) {
-            FAV_STAMP(ts, j, 0);
-            if (!fav::mbar_wait(s_full + 8 * i, j & 1, status)) { ok = false; break; }
-            FAV_STAMP(ts, j, 1);
-            fav::tc::fence_after();
-            const int key0 = j * BN;
-            const bool crosses = key0 + BN > lim_tile;   // tile crosses the diagonal or the end
-            float s[BN];
-            // S row from TMEM (and the mask: keys at or beyond lim get -inf)
-            auto load_s = [&]() {
-                uint32_t r[BN / 32][32];
+        for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
+            const Unit U = make_unit(u);
+            const int n_mine = U.n_kv_tiles[i];
+            if (n_mine == 0) continue;
+            const int ti = U.t[i], hi = U.h[i];
+            const int q0 = ti * BM;
+            const int qi = q0 + row;                          // query index of this row
+            const int lim = causal ? min(Nkv, qi + off + 1) : Nkv;       // visible keys: [0, lim)
+            const int lim_tile = causal ? min(Nkv, q0 + off + 1) : Nkv;  // smallest lim in the tile
+            float m = -INFINITY, l = 0.f;
+            for (int j = 0; j < n_mine; ++j) {
+                if (k == 0) FAV_STAMP(ts, j, 0);
+                if (!__all_sync(~0u, fav::mbar_wait(s_full + 8 * i, ns & 1, status))) { ok = false; break; }
+                ++ns;
+                if (k == 0) FAV_STAMP(ts, j, 1);
+                fav::tc::fence_after();
+                const int key0 = j * BN;
+                const bool crosses = key0 + BN > lim_tile;   // tile crosses the diagonal or the end
+                float s[BN];
+                // S row from TMEM (and the mask: keys at or beyond lim get -inf)
+                auto load_s = [&]() {
+                    uint32_t r[BN / 32][32];
 #pragma unroll
-                for (int c = 0; c < BN / 32; ++c) fav::tc::ld_32x32b_x32(trow + colS + c * 32, r[c]);
+                    for (int c = 0; c < BN / 32; ++c) fav::tc::ld_32x32b_x32(trow + colS + c * 32, r[c]);
 #pragma unroll
-                for (int c = 0; c < BN / 32; ++c) fav::tc::wait_ld_dep(r[c]);
+                    for (int c = 0; c < BN / 32; ++c) fav::tc::wait_ld_dep(r[c]);
 #pragma unroll
-                for (int c = 0; c < BN; ++c) s[c] = __uint_as_float(r[c >> 5][c & 31]);
-                if (crosses) {
+                    for (int c = 0; c < BN; ++c) s[c] = __uint_as_float(r[c >> 5][c & 31]);
+                    if (crosses) {
 #pragma unroll
-                    for (int c = 0; c < BN; ++c)
-                        if (key0 + c >= lim) s[c] = -INFINITY;
-                }
-            };
-            // raw row maximum: 8 independent chains of 3-input max, then a tree
-            auto row_max = [&]() {
-                float m8[8];
-#pragma unroll
-                for (int c = 0; c < 8; ++c) m8[c] = s[c];
-#pragma unroll
-                for (int c = 8; c < BN; c += 16) {
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) m8[k] = fav::fmax3(m8[k], s[c + k], s[c + 8 + k]);
-                }
-                return fav::fmax3(fav::fmax3(m8[0], m8[1], m8[2]), fav::fmax3(m8[3], m8[4], m8[5]),
-                                  fmaxf(m8[6], m8[7]));
-            };
-            // p = exp2(s * scale_log2 - mref) on pairs (one packed FMA, two ex2, one packed add),
-            // fp16 weights stored to TMEM half a row at a time (keys [64h, 64h + 64) over S
-            // columns [32h, 32h + 32), whose scores are already in registers); returns nothing,
-            // accumulates the fp32 sum in psum.
-            float psum = 0.f;
-            auto exp_store = [&](float mref) {
-                const float2 sc2 = make_float2(scale_log2, scale_log2);
-                const float2 nm2 = make_float2(-mref, -mref);
-                float2 l4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-                static_for<0, 2>([&](auto hc) {
-                    constexpr int h = decltype(hc)::value;
-                    uint32_t pk[32];
-                    static_for<0, 32>([&](auto pc) {
-                        constexpr int e = 2 * decltype(pc)::value;
-                        constexpr int c = 64 * h + e;
-                        const float2 x = fav::ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
-                        const float2 p = exp2_pair<c / 2>(x);
-                        l4[(e >> 1) & 3] = fav::fadd2(l4[(e >> 1) & 3], p);
-                        pk[e >> 1] = fav::Elem<TP>::pack(p.x, p.y);
-                    });
-                    fav::tc::st_32x32b_x32(trow + colS + 32 * h, pk);
-                });
-                const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
-                psum = a.x + a.y;
-            };
-            float alpha = 1.f;
-            bool rescale = false;
-            // lazy rescale: move the reference maximum only when it grows by > 2^8
-            auto move_max = [&](float mx) {
-                if (mx > m + kRescaleThreshold) {
-                    alpha = fav::fast_exp2(m - mx);   // 0 on the first tile (m = -inf)
-                    rescale = (j > 0);
-                    m = mx;
-                    l *= alpha;
-                }
-            };
-            // two passes: the row maximum, then the weights against the (lazy) reference
-            load_s();
-            FAV_STAMP(ts, j, 2);
-            move_max(row_max() * scale_log2);
-            FAV_STAMP(ts, j, 3);
-            // P_i over the first 64 columns of S_i (two 16-bit weights per column)
-            exp_store(m - kPShift);
-            l += psum;
-            FAV_STAMP(ts, j, 4);
-            // O_i is stable here: P_i(j-1).V completed before S_i(j) (in-order MMAs, one commit).
-            if (__any_sync(~0u, rescale)) {
-#pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    const uint32_t col = colO + c * 32;
-                    uint32_t v[32];
-                    fav::tc::ld_32x32b_x32(trow + col, v);
-                    fav::tc::wait_ld_dep(v);
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        const float2 y = fav::fmul2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])),
-                                                    make_float2(alpha, alpha));
-                        v[e] = __float_as_uint(y.x);
-                        v[e + 1] = __float_as_uint(y.y);
+                        for (int c = 0; c < BN; ++c)
+                            if (key0 + c >= lim) s[c] = -INFINITY;
                     }
-                    fav::tc::st_32x32b_x32(trow + col, v);
+                };
+                // raw row maximum: 8 independent chains of 3-input max, then a tree
+                auto row_max = [&]() {
+                    float m8[8];
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) m8[c] = s[c];
+#pragma unroll
+                    for (int c = 8; c < BN; c += 16) {
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) m8[q] = fav::fmax3(m8[q], s[c + q], s[c + 8 + q]);
+                    }
+                    return fav::fmax3(fav::fmax3(m8[0], m8[1], m8[2]), fav::fmax3(m8[3], m8[4], m8[5]),
+                                      fmaxf(m8[6], m8[7]));
+                };
+                // p = exp2(s * scale_log2 - mref) on pairs (one packed FMA, two ex2, one packed
+                // add), fp16 weights stored to TMEM half a row at a time (keys [64h, 64h + 64)
+                // over S columns [32h, 32h + 32), whose scores are already in registers); the
+                // fp32 sum goes to psum.
+                float psum = 0.f;
+                auto exp_store = [&](float mref) {
+                    const float2 sc2 = make_float2(scale_log2, scale_log2);
+                    const float2 nm2 = make_float2(-mref, -mref);
+                    float2 l4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+                    static_for<0, 2>([&](auto hc) {
+                        constexpr int h = decltype(hc)::value;
+                        uint32_t pk[32];
+                        static_for<0, 32>([&](auto pc) {
+                            constexpr int e = 2 * decltype(pc)::value;
+                            constexpr int c = 64 * h + e;
+                            const float2 x = fav::ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
+                            const float2 p = exp2_pair<c / 2>(x);
+                            l4[(e >> 1) & 3] = fav::fadd2(l4[(e >> 1) & 3], p);
+                            pk[e >> 1] = fav::Elem<TP>::pack(p.x, p.y);
+                        });
+                        fav::tc::st_32x32b_x32(trow + colS + 32 * h, pk);
+                    });
+                    const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
+                    psum = a.x + a.y;
+                };
+                float alpha = 1.f;
+                bool rescale = false;
+                // lazy rescale: move the reference maximum only when it grows by > 2^4
+                auto move_max = [&](float mx) {
+                    if (mx > m + kRescaleThreshold) {
+                        alpha = fav::fast_exp2(m - mx);   // 0 on the first tile (m = -inf)
+                        rescale = (j > 0);
+                        m = mx;
+                        l *= alpha;
+                    }
+                };
+                // two passes: the row maximum, then the weights against the (lazy) reference
+                load_s();
+                if (k == 0) FAV_STAMP(ts, j, 2);
+                move_max(row_max() * scale_log2);
+                if (k == 0) FAV_STAMP(ts, j, 3);
+                // P_i over the first 64 columns of S_i (two 16-bit weights per column)
+                exp_store(m - kPShift);
+                l += psum;
+                if (k == 0) FAV_STAMP(ts, j, 4);
+                // O_i is stable here: P_i(j-1).V completed before S_i(j) (in-order MMAs, one commit).
+                if (__any_sync(~0u, rescale)) {
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        const uint32_t col = colO + c * 32;
+                        uint32_t v[32];
+                        fav::tc::ld_32x32b_x32(trow + col, v);
+                        fav::tc::wait_ld_dep(v);
+#pragma unroll
+                        for (int e = 0; e < 32; e += 2) {
+                            const float2 y = fav::fmul2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])),
+                                                        make_float2(alpha, alpha));
+                            v[e] = __float_as_uint(y.x);
+                            v[e + 1] = __float_as_uint(y.y);
+                        }
+                        fav::tc::st_32x32b_x32(trow + col, v);
+                    }
                 }
+                fav::tc::wait_st();
+                fav::tc::fence_before();
+                __syncwarp();
+                if (lane == 0) fav::mbar_arrive(p_full + 8 * i);
+                if (k == 0) FAV_STAMP(ts, j, 5);
             }
-            fav::tc::wait_st();
-            fav::tc::fence_before();
-            __syncwarp();
-            if (lane == 0) fav::mbar_arrive(p_full + 8 * i);
-            FAV_STAMP(ts, j, 5);
-        }
 #ifdef FAV_TIMING
-        if (blockIdx.x == 0 && lane == 0 && n_mine > 5)
-            printf("[w%d j5] wait %6lld s_ready %6lld ld %6lld spec %6lld chk %6lld arrive %6lld\n", warp,
-                   ts[5][0] - t_start, ts[5][1] - t_start, ts[5][2] - t_start, ts[5][3] - t_start,
-                   ts[5][4] - t_start, ts[5][5] - t_start);
-        if (blockIdx.x == 0 && (threadIdx.x & 127) == 0)
-            for (int j = 0; j < min(n_mine, 16); ++j)
-                printf("[sm%d] j=%2d wait %6lld s_ready %6lld ld %6lld max %6lld exp %6lld arrive %6lld\n",
-                       i, j, ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start,
-                       ts[j][3] - t_start, ts[j][4] - t_start, ts[j][5] - t_start);
+            if (k == 0 && blockIdx.x == 0 && (threadIdx.x & 127) == 0)
+                for (int j = 0; j < min(n_mine, 16); ++j)
+                    printf("[sm%d] j=%2d wait %6lld s_ready %6lld ld %6lld max %6lld exp %6lld arrive %6lld\n",
+                           i, j, ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start,
+                           ts[j][3] - t_start, ts[j][4] - t_start, ts[j][5] - t_start);
 #endif
-        // ---------------- epilogue: O / l, LSE ----------------
-        if (ok && n_mine > 0 && fav::mbar_wait(o_done + 8 * i, 0, status)) {
+            if (!ok) break;
+            // ---------------- epilogue: O / l, LSE ----------------
+            // (the next unit's first P.V, which overwrites O_i, waits for this warpgroup's next
+            // P_i: it cannot run before these loads)
+            if (!__all_sync(~0u, fav::mbar_wait(o_done + 8 * i, no & 1, status))) { ok = false; break; }
+            ++no;
             fav::tc::fence_after();
+            const float vsc = kV16 ? v_scale[U.bkv] : 1.f;     // V = v_scale * (fp16 copy)
             const float inv_l = vsc / l;
             const bool valid = qi < Nq;
-            T *orow = o + ((long long)(b * Hq + hi) * Nq + qi) * D;
+            T *orow = o + ((long long)(U.b * Hq + hi) * Nq + qi) * D;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t v[32];
@@ -502,7 +547,8 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     }
                 }
             }
-            if (valid && lse) lse[(long long)(b * Hq + hi) * Nq + qi] = (m - kPShift + log2f(l)) * kLn2;
+            if (valid && lse) lse[(long long)(U.b * Hq + hi) * Nq + qi] = (m - kPShift + log2f(l)) * kLn2;
+            fav::tc::fence_before();
         }
     }
 
@@ -628,9 +674,11 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
     const int n_qtiles = (a.Nq + BM - 1) / BM;
     const int G = a.Hq / a.Hkv;
     const int pair_heads = (G % 2 == 0) ? 1 : 0;
-    const long long blocks = pair_heads ? (long long)n_qtiles * a.B * (a.Hq / 2)
-                                        : (long long)((n_qtiles + 1) / 2) * a.B * a.Hq;
-    if (blocks > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
+    const long long units = pair_heads ? (long long)n_qtiles * a.B * (a.Hq / 2)
+                                       : (long long)((n_qtiles + 1) / 2) * a.B * a.Hq;
+    if (units > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
+    // persistent: one CTA per SM at most, each working through its share of the units
+    const long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
     kern<<<(unsigned)blocks, kThreads, C::kSmemBytes, stream>>>(
         tmQ, tmK, tmV, (T *)a.o, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
         pair_heads, a.scale * kLog2e, a.causal, a.dev_status);
