@@ -106,14 +106,21 @@ template <int D> struct PrefillCfg {
     static constexpr int kOffK = kOffQ + 2 * kQBytes;
     static constexpr int kOffV = kOffK + kStages * kKVBytes;
     static constexpr int kOffBar = kOffV + kStages * kKVBytes;
-    static constexpr int kNumBars = 2 + 1 + 4 * kStages + 2 + 2 + 2;
+    static constexpr int kNumBars = 2 + 1 + 4 * kStages + 2 + 2 + 2 + 2 + 2;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
     static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
-    // TMEM columns: S0 | S1 | O0 | O1.  P_i (fp16) aliases the first 64 columns of S_i.
+    // TMEM columns.  D = 128: S0 | S1 | O0 | O1, and P_i (fp16, two weights per column)
+    // aliases the first 64 columns of S_i.  D = 64 (kSepP): S0 | S1 | P0 | P1 | O0 | O1, the
+    // weights have columns of their own, so the next scores of a tile can be computed while its
+    // softmax still works on the current ones.
+    static constexpr bool kSepP = (D == 64);
     static constexpr uint32_t kTmemCols = 512;
     static __host__ __device__ constexpr uint32_t colS(int i) { return i ? 128u : 0u; }
-    static __host__ __device__ constexpr uint32_t colO(int i) { return 256u + (i ? D : 0); }
-    static_assert(256 + 2 * D <= 512, "TMEM budget");
+    static __host__ __device__ constexpr uint32_t colP(int i) { return kSepP ? 256u + 64u * i : colS(i); }
+    static __host__ __device__ constexpr uint32_t colO(int i) {
+        return kSepP ? 384u + 64u * i : 256u + (i ? D : 0);
+    }
+    static_assert(kSepP ? 384 + 2 * D <= 512 : 256 + 2 * D <= 512, "TMEM budget");
 };
 
 // bf16 I/O (kV16): Q, K and O are bf16; V has been converted to fp16 (tmV, scaled per KV head
@@ -143,6 +150,8 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     const uint32_t s_full = v_empty + 8 * S;      // [2], one per query tile
     const uint32_t p_full = s_full + 16;          // [2]
     const uint32_t o_done = p_full + 16;          // [2]
+    const uint32_t s_free = o_done + 16;          // [2] (kSepP) the softmax has read S_i
+    const uint32_t p_free = s_free + 16;          // [2] (kSepP) P_i.V has completed
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffTmemSlot);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -212,6 +221,8 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             fav::mbar_init(s_full + 8 * i, 1);
             fav::mbar_init(p_full + 8 * i, 4);
             fav::mbar_init(o_done + 8 * i, 1);
+            fav::mbar_init(s_free + 8 * i, 4);
+            fav::mbar_init(p_free + 8 * i, 1);
         }
         fav::mbar_fence_init();
     }
@@ -292,7 +303,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         // O_i (+)= P_i V, with P_i read from TMEM (8 columns = 16 keys per k-step) and V MN-major
         // in shared memory (8-key groups 1024 B apart, 64-column blocks one box apart).
         auto issue_pv = [&](int i, int st, uint32_t acc, uint32_t bar_a, uint32_t bar_b) {
-            fav::tc::mma_ts_burst_k128(tmem + C::colO(i), tmem + C::colS(i),
+            fav::tc::mma_ts_burst_k128(tmem + C::colO(i), tmem + C::colP(i),
                                        dv0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_pv, acc,
                                        bar_a, bar_b);
         };
@@ -311,10 +322,73 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
 #endif
         int g = 0;                 // key tiles streamed so far (ring sequence)
         int np[2] = {0, 0};        // P_i(.) consumed so far, per tile (p_full parity)
+        int nsi[2] = {0, 0};       // S_i(.) issued so far, per tile (s_free parity, kSepP)
         bool ok = true;
         for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
             const Unit U = make_unit(u);
             const int g0 = g;
+            if constexpr (C::kSepP) {
+                // Weights in their own columns: S_i(j+1) is issued as soon as the softmax has
+                // read S_i(j) (s_free), before P_i(j).V, which is issued when P_i(j) is ready;
+                // the softmax waits for P_i(j).V (p_free) before it stores P_i(j+1) or rescales
+                // O_i.  Each tile's softmax can then run from one key tile to the next without
+                // waiting for the tensor core.
+                const int last0 = U.n_kv_tiles[1] > 0 ? 1 : 0;      // last tile with work
+                if (!(ok = wait_all(k_full + 8 * (g0 % S), (g0 / S) & 1))) break;
+                // S_1(0) waits until tile 0's softmax has reached its exponentials: the two
+                // softmaxes then run half a period apart, so that one's exponentials (MUFU) overlap
+                // the other's loads and maxima instead of competing for the MUFU in lockstep;
+                // the offset carries over to the following key tiles.
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (U.n_kv_tiles[i] == 0) continue;
+                    if (!(ok = wait_all(q_full + 8 * i, k & 1))) break;
+                    if (i == 1 && !(ok = wait_all(s_free, (nsi[0] - 1) & 1))) break;
+                    if (nsi[i] > 0 && !(ok = wait_all(s_free + 8 * i, (nsi[i] - 1) & 1))) break;
+                    fav::tc::fence_after();
+                    issue_s(i, g0 % S, s_full + 8 * i, i == last0 ? k_empty + 8 * (g0 % S) : 0u);
+                    ++nsi[i];
+                }
+                if (!ok) break;
+                if (U.n_kv == 1) fav::tc::commit_elect(q_empty);    // no further S in this unit
+                for (int j = 0; ok && j < U.n_kv; ++j) {
+                    const int gj = g0 + j;
+                    const int st = gj % S, st1 = (gj + 1) % S;
+                    if (j + 1 < U.n_kv) {
+                        // the next scores, K_{j+1} released by the last tile's burst
+                        const int last1 = j + 1 < U.n_kv_tiles[1] ? 1 : 0;
+                        if (!(ok = wait_all(k_full + 8 * st1, ((gj + 1) / S) & 1))) break;
+#pragma unroll
+                        for (int i = 0; i < 2; ++i) {
+                            if (j + 1 >= U.n_kv_tiles[i]) continue;
+                            if (k == 0) FAV_STAMP(ts, j, 3 * i);
+                            if (!(ok = wait_all(s_free + 8 * i, (nsi[i] - 1) & 1))) break;
+                            fav::tc::fence_after();
+                            issue_s(i, st1, s_full + 8 * i, i == last1 ? k_empty + 8 * st1 : 0u);
+                            ++nsi[i];
+                        }
+                        if (!ok) break;
+                        // after the unit's last scores, its Q buffers can be refilled
+                        if (j + 2 == U.n_kv) fav::tc::commit_elect(q_empty);
+                    }
+                    // P_i(j).V_j, V_j released by the last tile's burst
+                    const int last = j < U.n_kv_tiles[1] ? 1 : 0;
+                    if (!(ok = wait_all(v_full + 8 * st, (gj / S) & 1))) break;
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) {
+                        if (j >= U.n_kv_tiles[i]) continue;
+                        if (!(ok = wait_all(p_full + 8 * i, np[i] & 1))) break;
+                        ++np[i];
+                        if (k == 0) FAV_STAMP(ts, j, 3 * i + 1);
+                        fav::tc::fence_after();
+                        issue_pv(i, st, j > 0 ? 1u : 0u, p_free + 8 * i, i == last ? v_empty + 8 * st : 0u);
+                        if (j + 1 == U.n_kv_tiles[i]) fav::tc::commit_elect(o_done + 8 * i);
+                        if (k == 0) FAV_STAMP(ts, j, 3 * i + 2);
+                    }
+                }
+                g += U.n_kv;
+                continue;
+            }
             // first scores of the unit (the previous unit's last P.V are ahead in the pipe, so
             // S_i(0) cannot overwrite its P_i before it is read)
             const int last0 = U.n_kv_tiles[1] > 0 ? 1 : 0;      // last tile with work
@@ -391,6 +465,8 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         const uint32_t colS = i ? C::colS(1) : C::colS(0);
         const uint32_t colO = i ? C::colO(1) : C::colO(0);
         int ns = 0, no = 0;        // S_i(.) and O_i completions consumed so far (parities)
+        int npst = 0;              // P_i(.) stored so far (kSepP: p_free parity)
+        const uint32_t colP = i ? C::colP(1) : C::colP(0);
         bool ok = true;
 #ifdef FAV_TIMING
         long long ts[16][6];
@@ -463,7 +539,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                             l4[(e >> 1) & 3] = fav::fadd2(l4[(e >> 1) & 3], p);
                             pk[e >> 1] = fav::Elem<TP>::pack(p.x, p.y);
                         });
-                        fav::tc::st_32x32b_x32(trow + colS + 32 * h, pk);
+                        fav::tc::st_32x32b_x32(trow + colP + 32 * h, pk);
                     });
                     const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
                     psum = a.x + a.y;
@@ -484,11 +560,28 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                 if (k == 0) FAV_STAMP(ts, j, 2);
                 move_max(row_max() * scale_log2);
                 if (k == 0) FAV_STAMP(ts, j, 3);
+                if constexpr (C::kSepP) {
+                    // S_i has been read (long ago; the signal waits for the start of the
+                    // exponentials, which also paces the other tile: see the MMA warp)
+                    fav::tc::fence_before();
+                    __syncwarp();
+                    if (lane == 0) fav::mbar_arrive(s_free + 8 * i);
+                }
                 // P_i over the first 64 columns of S_i (two 16-bit weights per column)
+                if constexpr (C::kSepP) {
+                    // P_i's columns and O_i are free and stable once the previous P_i.V is done
+                    if (npst > 0 && !__all_sync(~0u, fav::mbar_wait(p_free + 8 * i, (npst - 1) & 1, status))) {
+                        ok = false;
+                        break;
+                    }
+                    fav::tc::fence_after();
+                }
+                ++npst;
                 exp_store(m - kPShift);
                 l += psum;
                 if (k == 0) FAV_STAMP(ts, j, 4);
-                // O_i is stable here: P_i(j-1).V completed before S_i(j) (in-order MMAs, one commit).
+                // O_i is stable here: P_i(j-1).V has completed (D = 128: it was issued before
+                // S_i(j) and MMAs complete in issue order; D = 64: the p_free wait above).
                 if (__any_sync(~0u, rescale)) {
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
