@@ -351,40 +351,43 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                 }
                 if (!ok) break;
                 if (U.n_kv == 1) fav::tc::commit_elect(q_empty);    // no further S in this unit
+                // Per key tile j, tile by tile: S_i(j+1) (once the softmax has read S_i(j)), then
+                // P_i(j).V_j (once P_i(j) is stored).  Tile 1's softmax runs half a period behind
+                // tile 0's, so this order never holds one tile's MMAs behind the other's events.
+                // K_{j+1} and V_j are released by the last tile's bursts.
                 for (int j = 0; ok && j < U.n_kv; ++j) {
                     const int gj = g0 + j;
                     const int st = gj % S, st1 = (gj + 1) % S;
-                    if (j + 1 < U.n_kv) {
-                        // the next scores, K_{j+1} released by the last tile's burst
-                        const int last1 = j + 1 < U.n_kv_tiles[1] ? 1 : 0;
-                        if (!(ok = wait_all(k_full + 8 * st1, ((gj + 1) / S) & 1))) break;
+                    const int last1 = j + 1 < U.n_kv_tiles[1] ? 1 : 0;   // last tile with S(j+1)
+                    const int last = j < U.n_kv_tiles[1] ? 1 : 0;        // last tile with P(j)
+                    bool k_ok = false, v_ok = false;
 #pragma unroll
-                        for (int i = 0; i < 2; ++i) {
-                            if (j + 1 >= U.n_kv_tiles[i]) continue;
+                    for (int i = 0; i < 2; ++i) {
+                        if (j + 1 < U.n_kv_tiles[i]) {
+                            if (!k_ok && !(ok = wait_all(k_full + 8 * st1, ((gj + 1) / S) & 1))) break;
+                            k_ok = true;
                             if (k == 0) FAV_STAMP(ts, j, 3 * i);
                             if (!(ok = wait_all(s_free + 8 * i, (nsi[i] - 1) & 1))) break;
                             fav::tc::fence_after();
                             issue_s(i, st1, s_full + 8 * i, i == last1 ? k_empty + 8 * st1 : 0u);
                             ++nsi[i];
                         }
-                        if (!ok) break;
-                        // after the unit's last scores, its Q buffers can be refilled
-                        if (j + 2 == U.n_kv) fav::tc::commit_elect(q_empty);
+                        if (j < U.n_kv_tiles[i]) {
+                            if (!v_ok && !(ok = wait_all(v_full + 8 * st, (gj / S) & 1))) break;
+                            v_ok = true;
+                            if (!(ok = wait_all(p_full + 8 * i, np[i] & 1))) break;
+                            ++np[i];
+                            if (k == 0) FAV_STAMP(ts, j, 3 * i + 1);
+                            fav::tc::fence_after();
+                            issue_pv(i, st, j > 0 ? 1u : 0u, p_free + 8 * i, i == last ? v_empty + 8 * st : 0u);
+                            if (j + 1 == U.n_kv_tiles[i]) fav::tc::commit_elect(o_done + 8 * i);
+                            if (k == 0) FAV_STAMP(ts, j, 3 * i + 2);
+                        }
                     }
-                    // P_i(j).V_j, V_j released by the last tile's burst
-                    const int last = j < U.n_kv_tiles[1] ? 1 : 0;
-                    if (!(ok = wait_all(v_full + 8 * st, (gj / S) & 1))) break;
-#pragma unroll
-                    for (int i = 0; i < 2; ++i) {
-                        if (j >= U.n_kv_tiles[i]) continue;
-                        if (!(ok = wait_all(p_full + 8 * i, np[i] & 1))) break;
-                        ++np[i];
-                        if (k == 0) FAV_STAMP(ts, j, 3 * i + 1);
-                        fav::tc::fence_after();
-                        issue_pv(i, st, j > 0 ? 1u : 0u, p_free + 8 * i, i == last ? v_empty + 8 * st : 0u);
-                        if (j + 1 == U.n_kv_tiles[i]) fav::tc::commit_elect(o_done + 8 * i);
-                        if (k == 0) FAV_STAMP(ts, j, 3 * i + 2);
-                    }
+                    if (!ok) break;
+                    // after the unit's last scores (issued in this key tile), its Q buffers can be
+                    // refilled: the commit covers every MMA issued so far
+                    if (j + 2 == U.n_kv) fav::tc::commit_elect(q_empty);
                 }
                 g += U.n_kv;
                 continue;
