@@ -7,33 +7,35 @@
 // block the accumulator is normalised.  Heads sharing a K/V head read the same K/V tiles
 // (GQA reuse), and several heads are processed by one unit of work (the paper's inter-head
 // parallelism).  On this GPU that becomes:
-//   * each CTA owns two 128-row query tiles that read the same K/V head: the same query tile
-//     of two heads of one GQA group (even group sizes), or two consecutive query tiles of one
-//     head (MHA).  Both Q tiles live in shared memory (TMA, 128-byte swizzle), loaded once;
+//   * a unit is two 128-row query tiles that read the same K/V head: the same query tile of
+//     two heads of one GQA group (even group sizes), or two consecutive query tiles of one
+//     head.  The kernel is persistent (one CTA per SM at most); CTA c works through units
+//     c, 2P-1-c, 2P+c, ... of the units sorted by decreasing causal work, loading the next
+//     unit's Q tiles (TMA, 128-byte swizzle) during the current unit's tail;
 //   * 128-key K and V tiles are streamed by TMA through a ring of shared-memory stages and
 //     serve both query tiles;
 //   * S_i = Q_i K^T (M = 128, N = 128, K = D) and O_i += P_i V (M = 128, N = D, K = 128) are
 //     bursts of tcgen05.mma issued by one elected lane of a converged warp, accumulating in
-//     tensor memory (TMEM).  P_i is written
-//     back into TMEM over the columns of S_i and read from there by the P.V MMA;
+//     tensor memory (TMEM), with P_i read from TMEM;
 //   * one softmax warpgroup per query tile, one thread per query row (= TMEM lane): tcgen05.ld
-//     of its S row, mask, row max, exp2 in the log2 domain, row sum, P rounded to the I/O type,
-//     tcgen05.st of P.  The MMA thread alternates between the two tiles (P.V and the next
-//     Q.K^T of tile 0 while the softmax works on tile 1, and vice versa), so the tensor core
-//     and the softmax overlap.
+//     of its scores, mask, row maximum, exp2 in the log2 domain, row sum, fp16 weights stored
+//     with tcgen05.st.
+// D = 128: TMEM holds S0 | S1 | O0 | O1 and P_i overwrites the first half of S_i, so S_i(j+1)
+// can only follow P_i(j).V; the MMA warp alternates [P_0(j).V, S_0(j+1)], [P_1(j).V, S_1(j+1)]
+// and each softmax runs while the tensor core works on the other tile.  D = 64: the weights
+// have columns of their own (S0 | S1 | P0 | P1 | O0 | O1), S_i(j+1) is issued as soon as the
+// softmax has read S_i(j), and the two tiles' softmaxes run back to back, half a period apart.
 // The running maximum is updated lazily: O and l are rescaled only when the maximum grows by
-// more than 2^8 (log2 domain); otherwise the stale maximum is kept and the weights may reach
-// 256.  The final O / l uses the same maximum as every weight, so the result is unchanged.
-// Because MMAs complete in issue order and S_i(j) is issued after P_i(j-1).V, O_i is stable
-// when S_i(j) arrives: the softmax thread rescales it itself, before writing P_i(j).
+// more than 2^4 (log2 domain); the weights are stored as p * 2^11 (below 2^15, inside fp16's
+// range).  The final O / l uses the same maximum as every weight, so the result is unchanged.
 //
 // Warp roles (320 threads): warps 0-3 softmax of tile 0, warps 4-7 softmax of tile 1
 // (TMEM lane quarter = warp % 4); warp 8 = TMEM owner + MMA issuer (the whole warp, one
-// elected lane issuing each burst); warp 9 = TMA producer.  The issuing lane blocks while the
-// tensor pipe is busy, and a wait on an mbarrier costs ~80 cycles of latency even when the
-// phase is already complete; so the warp tests the barriers it will need next *before* a
-// burst of MMAs and looks at the answers after it, and only waits for real on the ones that
-// were not complete.
+// elected lane issuing each burst and committing the barrier arrivals inside the same asm
+// block); warp 9 = TMA producer.  The issuing lane blocks while the tensor pipe is busy, and a
+// wait on an mbarrier costs ~80 cycles of latency even when the phase is already complete; so
+// the warp tests the barriers it will need next *before* a burst of MMAs where it can, and
+// only waits for real on the ones that were not complete.
 #include <cuda.h>
 #include <math.h>
 
