@@ -86,6 +86,38 @@ FAV_API fav_status fav_forward(const void *q, const void *k, const void *v, void
                        float scale, int causal, fav_dtype dtype, void *stream);
 
 /*
+ * Element strides of a [B, H, N, D] tensor whose D axis is contiguous: the distance, in
+ * elements, between consecutive batches, heads and tokens.  The contiguous layout is
+ * {H * N * D, N * D, D}; the heads-interleaved layout [B, N, H, D] (one token's heads stored
+ * together) is {N * H * D, D, H * D}; a padded or sliced cache has larger token strides.
+ */
+typedef struct {
+    long long batch, head, token;
+} fav_strides;
+
+/*
+ * fav_forward_strided -- fav_forward on tensors given by their strides.  (Method section,
+ * optimizations for VL > D: in the ggml memory layout the paper works on, the heads of one
+ * token lie next to each other, [B, N, H, D], and its kernel reorders the loop over heads to
+ * read that layout directly.  This entry point takes that layout, and any other with a
+ * contiguous D axis, without copies.)
+ *
+ *  q, k, v, o   device pointers to element (0, 0, 0, 0), 16-byte aligned
+ *  *_strides    element strides; each stride times the element size must be a multiple of 16
+ *               bytes and below 2^40, else FAV_ERR_UNSUPPORTED.  Negative strides:
+ *               FAV_ERR_INVALID_ARG.  A stride of 0 is accepted only on an axis of size 1
+ *               (o: FAV_ERR_INVALID_ARG otherwise; q, k, v: FAV_ERR_UNSUPPORTED).  Distinct
+ *               rows of o must not overlap (not checked otherwise).
+ *  lse          [B, Hq, Nq] fp32, contiguous, or NULL
+ *  other arguments and statuses as fav_forward; the call is asynchronous on `stream`.
+ */
+FAV_API fav_status fav_forward_strided(const void *q, const void *k, const void *v, void *o,
+                                       float *lse, fav_strides q_strides, fav_strides k_strides,
+                                       fav_strides v_strides, fav_strides o_strides, int B,
+                                       int Hq, int Hkv, int Nq, int Nkv, int D, float scale,
+                                       int causal, fav_dtype dtype, void *stream);
+
+/*
  * fav_forward_host -- the same operation on HOST buffers (end-to-end call).
  *
  * Copies q, k, v (host, ideally pinned) to internal device buffers, computes, copies o and lse

@@ -7,7 +7,7 @@ CPU fallback: without the built library every call raises.
 import ctypes
 import os
 
-__all__ = ["forward", "forward_host", "set_path", "last_path", "set_decode_splits",
+__all__ = ["forward", "forward_host", "Strides", "set_path", "last_path", "set_decode_splits",
            "last_decode_splits", "device_status", "release_workspace", "library_path",
            "FavError", "F32", "F16", "BF16", "PATH_AUTO", "PATH_SIMT", "PATH_DECODE",
            "PATH_PREFILL"]
@@ -22,6 +22,12 @@ STATUS_NAMES = {0: "FAV_OK", 1: "FAV_ERR_INVALID_ARG", 2: "FAV_ERR_UNSUPPORTED",
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "libfav.so")
 _lib = None
+
+
+class Strides(ctypes.Structure):
+    """fav_strides: element strides (batch, head, token) of a [B, H, N, D] tensor."""
+    _fields_ = [("batch", ctypes.c_longlong), ("head", ctypes.c_longlong),
+                ("token", ctypes.c_longlong)]
 
 
 class FavError(RuntimeError):
@@ -47,6 +53,10 @@ def lib():
         for fn in ("fav_forward", "fav_forward_host"):
             getattr(L, fn).argtypes = sig
             getattr(L, fn).restype = i
+        S = Strides
+        L.fav_forward_strided.argtypes = [vp, vp, vp, vp, vp, S, S, S, S, i, i, i, i, i, i,
+                                          ctypes.c_float, i, i, vp]
+        L.fav_forward_strided.restype = i
         L.fav_status_string.argtypes = [i]
         L.fav_status_string.restype = ctypes.c_char_p
         L.fav_get_last_device_status.argtypes = []
@@ -82,15 +92,18 @@ def forward(q, k, v, causal=False, scale=None, return_lse=True, out=None, lse_ou
             stream=None):
     """Attention forward on torch CUDA tensors q [B,Hq,Nq,D], k/v [B,Hkv,Nkv,D].
 
-    Returns (o, lse) with lse [B,Hq,Nq] fp32 (None if return_lse is False).  Runs on the
-    current torch stream unless ``stream`` (a torch.cuda.Stream) is given.
+    The tensors may be any strided views whose last axis is contiguous (for example
+    ``x.transpose(1, 2)`` of a [B, N, H, D] tensor): those go through fav_forward_strided.
+    Returns (o, lse) with lse [B,Hq,Nq] fp32 (None if return_lse is False); o is allocated
+    contiguous unless ``out`` is given.  Runs on the current torch stream unless ``stream``
+    (a torch.cuda.Stream) is given.
     """
     import torch
     for t in (q, k, v):
         if not t.is_cuda:
             raise ValueError("tensors must live on a CUDA device")
-        if not t.is_contiguous():
-            raise ValueError("tensors must be contiguous")
+        if t.dim() != 4 or t.stride(-1) != 1:
+            raise ValueError("tensors must be 4-D with a contiguous last axis")
     if k.dtype != q.dtype or v.dtype != q.dtype:
         raise TypeError("q, k and v must share a dtype")
     B, Hq, Nq, D = q.shape
@@ -100,17 +113,26 @@ def forward(q, k, v, causal=False, scale=None, return_lse=True, out=None, lse_ou
     if scale is None:
         import numpy as np
         scale = float(np.float32(1.0 / np.sqrt(D)))
-    o = out if out is not None else torch.empty_like(q)
+    o = out if out is not None else torch.empty(q.shape, dtype=q.dtype, device=q.device)
+    if o.dim() != 4 or o.stride(-1) != 1:
+        raise ValueError("out must be 4-D with a contiguous last axis")
     lse = None
     if return_lse:
         lse = lse_out if lse_out is not None else torch.empty((B, Hq, Nq), device=q.device,
                                                               dtype=torch.float32)
     s = stream if stream is not None else torch.cuda.current_stream(q.device)
+    lse_ptr = lse.data_ptr() if lse is not None else None
     with torch.cuda.device(q.device):
-        st = lib().fav_forward(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(),
-                               lse.data_ptr() if lse is not None else None, B, Hq, Hkv, Nq,
-                               Nkv, D, float(scale), int(bool(causal)), _dtype_code(q),
-                               s.cuda_stream)
+        if all(t.is_contiguous() for t in (q, k, v, o)):
+            st = lib().fav_forward(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(),
+                                   lse_ptr, B, Hq, Hkv, Nq, Nkv, D, float(scale),
+                                   int(bool(causal)), _dtype_code(q), s.cuda_stream)
+        else:
+            sd = [Strides(t.stride(0), t.stride(1), t.stride(2)) for t in (q, k, v, o)]
+            st = lib().fav_forward_strided(q.data_ptr(), k.data_ptr(), v.data_ptr(),
+                                           o.data_ptr(), lse_ptr, *sd, B, Hq, Hkv, Nq, Nkv, D,
+                                           float(scale), int(bool(causal)), _dtype_code(q),
+                                           s.cuda_stream)
     _check(st)
     return o, lse
 

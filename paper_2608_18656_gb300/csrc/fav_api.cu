@@ -85,6 +85,8 @@ FavArgs make_args(const void *q, const void *k, const void *v, void *o, float *l
                   int Hkv, int Nq, int Nkv, int D, float scale, int causal, fav_dtype dtype) {
     FavArgs a;
     a.q = q; a.k = k; a.v = v; a.o = o; a.lse = lse;
+    a.qs = a.os = fav_contiguous_strides(Hq, Nq, D);
+    a.ks = a.vs = fav_contiguous_strides(Hkv, Nkv, D);
     a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.Nq = Nq; a.Nkv = Nkv; a.D = D;
     a.scale = scale; a.causal = causal; a.dtype = dtype;
     a.dev_status = nullptr;
@@ -210,7 +212,8 @@ bool fav_debug_sync(const char *what, cudaStream_t s) {
     return e != cudaSuccess;
 }
 
-fav_status fav_make_tmap_3d(void *tmap, const void *base, int D, int rows, int outer, int box_rows) {
+fav_status fav_make_tmap_4d(void *tmap, const void *base, int D, int rows, int heads, int batch,
+                            FavStrides st, int box_rows) {
     static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     static std::once_flag once;
     std::call_once(once, [] {
@@ -222,11 +225,18 @@ fav_status fav_make_tmap_3d(void *tmap, const void *base, int D, int rows, int o
             encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     });
     if (!encode) return FAV_ERR_CUDA;
-    const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)outer};
-    const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)rows * D * 2};
-    const cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
-    const cuuint32_t estr[3] = {1, 1, 1};
-    CUresult r = encode(reinterpret_cast<CUtensorMap *>(tmap), CU_TENSOR_MAP_DATA_TYPE_UINT16, 3,
+    const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)heads,
+                                (cuuint64_t)batch};
+    // A stride of 0 is only accepted on an axis of size 1 (validation), where only coordinate 0
+    // is ever read: it gets a nominal nonzero stride for the encoder.
+    auto bstride = [](long long e, long long fallback) {
+        return (cuuint64_t)((e > 0 ? e : fallback) * 2);
+    };
+    const cuuint64_t strides[3] = {bstride(st.n, D), bstride(st.h, (long long)rows * D),
+                                   bstride(st.b, (long long)heads * rows * D)};
+    const cuuint32_t box[4] = {64, (cuuint32_t)box_rows, 1, 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = encode(reinterpret_cast<CUtensorMap *>(tmap), CU_TENSOR_MAP_DATA_TYPE_UINT16, 4,
                         const_cast<void *>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -245,6 +255,44 @@ fav_status fav_forward(const void *q, const void *k, const void *v, void *o, flo
     fav_status st = validate_shape(B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
     if (st != FAV_OK) return st;
     const FavArgs a = make_args(q, k, v, o, lse, B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    return forward_impl(a, static_cast<cudaStream_t>(stream));
+}
+
+fav_status fav_forward_strided(const void *q, const void *k, const void *v, void *o, float *lse,
+                               fav_strides q_strides, fav_strides k_strides,
+                               fav_strides v_strides, fav_strides o_strides, int B, int Hq,
+                               int Hkv, int Nq, int Nkv, int D, float scale, int causal,
+                               fav_dtype dtype, void *stream) {
+    if (!q || !k || !v || !o) return FAV_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(o, 16))
+        return FAV_ERR_INVALID_ARG;
+    if (lse && !aligned(lse, 4)) return FAV_ERR_INVALID_ARG;
+    fav_status st = validate_shape(B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    if (st != FAV_OK) return st;
+    const long long es = dtype == FAV_F32 ? 4 : 2;
+    const fav_strides all[4] = {q_strides, k_strides, v_strides, o_strides};
+    for (const fav_strides &x : all) {
+        if (x.batch < 0 || x.head < 0 || x.token < 0) return FAV_ERR_INVALID_ARG;
+        // every row starts on a 16-byte boundary (vector loads, TMA), and TMA strides < 2^40 B
+        for (long long e : {x.batch, x.head, x.token})
+            if ((e * es) % 16 != 0 || e * es >= (1LL << 40)) return FAV_ERR_UNSUPPORTED;
+    }
+    // The output is written: its rows must not coincide (no zero stride on an axis longer than
+    // 1).  Inputs: broadcasting (zero stride on a longer axis) is not supported.
+    if ((o_strides.batch == 0 && B > 1) || (o_strides.head == 0 && Hq > 1) ||
+        (o_strides.token == 0 && Nq > 1))
+        return FAV_ERR_INVALID_ARG;
+    auto broadcast = [&](const fav_strides &x, int H, int N) {
+        return (x.batch == 0 && B > 1) || (x.head == 0 && H > 1) || (x.token == 0 && N > 1);
+    };
+    if (broadcast(q_strides, Hq, Nq) || broadcast(k_strides, Hkv, Nkv) || broadcast(v_strides, Hkv, Nkv))
+        return FAV_ERR_UNSUPPORTED;
+    FavArgs a = make_args(q, k, v, o, lse, B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    auto conv = [](const fav_strides &x) { return FavStrides{x.batch, x.head, x.token}; };
+    a.qs = conv(q_strides);
+    a.ks = conv(k_strides);
+    a.vs = conv(v_strides);
+    a.os = conv(o_strides);
     return forward_impl(a, static_cast<cudaStream_t>(stream));
 }
 

@@ -61,7 +61,8 @@ __device__ __forceinline__ uint32_t swz(int j, int c) {
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads, 1)
 fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                  const T *__restrict__ q, T *__restrict__ o, float *__restrict__ lse,
+                  const T *__restrict__ q, FavStrides qs, T *__restrict__ o, FavStrides os,
+                  float *__restrict__ lse,
                   float *__restrict__ part_o, float *__restrict__ part_lse, int Hq, int Hkv,
                   int Nq, int Nkv, int n_tiles, int tiles_per_split, int splits,
                   float scale_log2, int causal, int *status) {
@@ -129,8 +130,8 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
                                        ((kdst | vdst) & 1023u) == 0 && key0 < n_tiles * TK &&
                                        bkv < (int)gridDim.y, status))
                         continue;
-                    fav::tma_load_3d(kdst + bx * TK * 128, &tmK, full, bx * 64, key0, bkv);
-                    fav::tma_load_3d(vdst + bx * TK * 128, &tmV, full, bx * 64, key0, bkv);
+                    fav::tma_load_4d(kdst + bx * TK * 128, &tmK, full, bx * 64, key0, g, b);
+                    fav::tma_load_4d(vdst + bx * TK * 128, &tmV, full, bx * 64, key0, g, b);
                 }
             }
         }
@@ -147,7 +148,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         const int m = m0 + r + 8 * h2;
         if (m < M) {
             const int i = m / G, hh = m % G;
-            qrow[h2] = q + ((long long)(b * Hq + g * G + hh) * Nq + i) * D;
+            qrow[h2] = q + b * qs.b + (long long)(g * G + hh) * qs.h + (long long)i * qs.n;
             lim[h2] = causal ? (Nkv - Nq + i + 1) : Nkv;
         } else {
             qrow[h2] = nullptr;
@@ -333,7 +334,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     if (!FAV_CHECK(flat >= 0 && flat < rows_total && c0 + kCols <= D, status)) return;
     const float lse_val = (L > 0.f) ? (Mx + log2f(L)) * kLn2 : -INFINITY;
     if (splits == 1) {
-        T *orow = o + flat * D + c0;
+        T *orow = o + b * os.b + (long long)(g * G + hh) * os.h + (long long)i * os.n + c0;
 #pragma unroll
         for (int c = 0; c < kCols; c += 8) {
             uint4 pk;
@@ -361,7 +362,8 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
 template <typename T, int D>
 __global__ void __launch_bounds__(128)
 fav_combine_kernel(const float *__restrict__ part_o, const float *__restrict__ part_lse,
-                   T *__restrict__ o, float *__restrict__ lse, long long rows, int splits) {
+                   T *__restrict__ o, FavStrides os, int Hq, int Nq, float *__restrict__ lse,
+                   long long rows, int splits) {
     asm volatile("griddepcontrol.wait;" ::: "memory");
     __shared__ float red[4][D];
     __shared__ float wred[4];
@@ -414,7 +416,9 @@ fav_combine_kernel(const float *__restrict__ part_o, const float *__restrict__ p
         const int c = threadIdx.x * 2;
         const float x0 = red[0][c] + red[1][c] + red[2][c] + red[3][c];
         const float x1 = red[0][c + 1] + red[1][c + 1] + red[2][c + 1] + red[3][c + 1];
-        *reinterpret_cast<uint32_t *>(o + row * D + c) = fav::Elem<T>::pack(x0, x1);
+        const long long b = row / ((long long)Hq * Nq), h = (row / Nq) % Hq, i = row % Nq;
+        *reinterpret_cast<uint32_t *>(o + b * os.b + h * os.h + i * os.n + c) =
+            fav::Elem<T>::pack(x0, x1);
     }
     if (lse && threadIdx.x == 0) lse[row] = L;
 }
@@ -425,9 +429,9 @@ fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t st
     constexpr int TK = Cfg::TK;
     alignas(64) CUtensorMap tmK, tmV;
     const int outer = a.B * a.Hkv;
-    fav_status st = fav_make_tmap_3d(&tmK, a.k, D, a.Nkv, outer, TK);
+    fav_status st = fav_make_tmap_4d(&tmK, a.k, D, a.Nkv, a.Hkv, a.B, a.ks, TK);
     if (st != FAV_OK) return st;
-    st = fav_make_tmap_3d(&tmV, a.v, D, a.Nkv, outer, TK);
+    st = fav_make_tmap_4d(&tmV, a.v, D, a.Nkv, a.Hkv, a.B, a.vs, TK);
     if (st != FAV_OK) return st;
     const int n_tiles = fav_decode_num_tiles(a);
     const int tps = (n_tiles + splits - 1) / splits;
@@ -448,7 +452,7 @@ fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t st
     const float scale_log2 = a.scale * kLog2e;
     dim3 grid(splits, outer, chunks);
     kern<<<grid, kThreads, Cfg::kSmemBytes, stream>>>(
-        tmK, tmV, (const T *)a.q, (T *)a.o, a.lse, part_o, part_lse, a.Hq, a.Hkv, a.Nq, a.Nkv,
+        tmK, tmV, (const T *)a.q, a.qs, (T *)a.o, a.os, a.lse, part_o, part_lse, a.Hq, a.Hkv, a.Nq, a.Nkv,
         n_tiles, tps, splits, scale_log2, a.causal, a.dev_status);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_decode_kernel", stream))
         return FAV_ERR_CUDA;
@@ -467,7 +471,7 @@ fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t st
         T *out = (T *)a.o;
         float *lse_out = a.lse;
         cudaLaunchKernelEx(&cfg, fav_combine_kernel<T, D>, (const float *)part_o,
-                           (const float *)part_lse, out, lse_out, rows, splits);
+                           (const float *)part_lse, out, a.os, a.Hq, a.Nq, lse_out, rows, splits);
         if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_combine_kernel", stream))
             return FAV_ERR_CUDA;
     }

@@ -5,10 +5,16 @@
 
 #include "../../include/fav.h"
 
+// Element strides of a [B, H, N, D] tensor whose D axis is contiguous (batch, head, token).
+struct FavStrides {
+    long long b, h, n;
+};
+
 struct FavArgs {
     const void *q, *k, *v;
     void *o;
-    float *lse;
+    float *lse;                          // [B, Hq, Nq] contiguous
+    FavStrides qs, ks, vs, os;           // strides of q, k, v, o
     int B, Hq, Hkv, Nq, Nkv, D;
     float scale;
     int causal;
@@ -47,8 +53,14 @@ fav_status fav_internal_validate(int B, int Hq, int Hkv, int Nq, int Nkv, int D,
 fav_status fav_internal_device_info(int **dev_status, int *num_sms);
 int fav_internal_decode_splits_override();
 
+// Contiguous strides of a [B, H, N, D] tensor.
+inline FavStrides fav_contiguous_strides(int H, int N, int D) {
+    return FavStrides{(long long)H * N * D, (long long)N * D, (long long)D};
+}
+
 // Tensor-map encoding through the driver entry point (fav_api.cu).
-// 3-D map over a [outer, rows, D] tensor of 16-bit elements, box {64, box_rows, 1},
-// 128-byte swizzle, zero fill out of bounds.
-fav_status fav_make_tmap_3d(void *tmap /* CUtensorMap* */, const void *base, int D, int rows,
-                            int outer, int box_rows);
+// 4-D map over a [batch, heads, rows, D] tensor of 16-bit elements with element strides `st`
+// (D contiguous; the strides must be multiples of 8 elements), box {64, box_rows, 1, 1},
+// 128-byte swizzle, zero fill out of bounds.  Coordinates (x, row, head, batch).
+fav_status fav_make_tmap_4d(void *tmap /* CUtensorMap* */, const void *base, int D, int rows,
+                            int heads, int batch, FavStrides st, int box_rows);

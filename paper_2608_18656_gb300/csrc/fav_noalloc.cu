@@ -73,6 +73,8 @@ extern "C" FAV_API fav_status fav_decode_noalloc(const void *q, const void *k, c
     if (st != FAV_OK) return st;
     FavArgs a;
     a.q = q; a.k = k; a.v = v; a.o = o; a.lse = lse;
+    a.qs = a.os = fav_contiguous_strides(Hq, Nq, D);
+    a.ks = a.vs = fav_contiguous_strides(Hkv, Nkv, D);
     a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.Nq = Nq; a.Nkv = Nkv; a.D = D;
     a.scale = scale; a.causal = causal; a.dtype = dtype;
     if (!fav_decode_supported(a)) return FAV_ERR_UNSUPPORTED;

@@ -131,7 +131,7 @@ template <int D> struct PrefillCfg {
 template <typename T, int D, bool kV16>
 __global__ void __launch_bounds__(kThreads, 1)
 fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   const __grid_constant__ CUtensorMap tmV, T *__restrict__ o,
+                   const __grid_constant__ CUtensorMap tmV, T *__restrict__ o, FavStrides os,
                    float *__restrict__ lse, const float *__restrict__ v_scale, int B, int Hq,
                    int Hkv, int Nq, int Nkv, int n_qtiles, int pair_heads, float scale_log2,
                    int causal, int *status) {
@@ -166,7 +166,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     // (P CTAs, "snake" order): with the units sorted by decreasing work, this evens out the
     // sums per CTA.
     struct Unit {
-        int b, h[2], t[2], n_kv_tiles[2], n_kv, bkv;
+        int b, h[2], t[2], n_kv_tiles[2], n_kv, kvh, bkv;
     };
     const int n_units = pair_heads ? n_qtiles * B * (Hq / 2) : ((n_qtiles + 1) / 2) * B * Hq;
     auto unit_at = [&](int k) {   // the k-th unit of this CTA, or -1
@@ -193,7 +193,8 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             U.t[0] = 2 * pr;
             U.t[1] = 2 * pr + 1;
         }
-        U.bkv = U.b * Hkv + U.h[0] / G;
+        U.kvh = U.h[0] / G;
+        U.bkv = U.b * Hkv + U.kvh;
 #pragma unroll
         for (int i = 0; i < 2; ++i) {
             if (U.t[i] >= n_qtiles) {
@@ -263,8 +264,8 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     fav::mbar_arrive_expect_tx(q_full + 8 * i, C::kQBytes);
 #pragma unroll
                     for (int bx = 0; bx < C::kBoxes; ++bx)
-                        fav::tma_load_3d(sbase + C::kOffQ + i * C::kQBytes + bx * BM * 128, &tmQ,
-                                         q_full + 8 * i, bx * 64, U.t[i] * BM, U.b * Hq + U.h[i]);
+                        fav::tma_load_4d(sbase + C::kOffQ + i * C::kQBytes + bx * BM * 128, &tmQ,
+                                         q_full + 8 * i, bx * 64, U.t[i] * BM, U.h[i], U.b);
                 }
                 // Each stage has its own empty barriers (one commit per use, waited in order).
                 for (int j = 0; j < U.n_kv; ++j, ++g) {
@@ -274,14 +275,14 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                     fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
 #pragma unroll
                     for (int bx = 0; bx < C::kBoxes; ++bx)
-                        fav::tma_load_3d(sK + st * C::kKVBytes + bx * BN * 128, &tmK, k_full + 8 * st,
-                                         bx * 64, j * BN, U.bkv);
+                        fav::tma_load_4d(sK + st * C::kKVBytes + bx * BN * 128, &tmK, k_full + 8 * st,
+                                         bx * 64, j * BN, U.kvh, U.b);
                     if (g >= S && !fav::mbar_wait(v_empty + 8 * st, ph, status)) { ok = false; break; }
                     fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
 #pragma unroll
                     for (int bx = 0; bx < C::kBoxes; ++bx)
-                        fav::tma_load_3d(sV + st * C::kKVBytes + bx * BN * 128, &tmV, v_full + 8 * st,
-                                         bx * 64, j * BN, U.bkv);
+                        fav::tma_load_4d(sV + st * C::kKVBytes + bx * BN * 128, &tmV, v_full + 8 * st,
+                                         bx * 64, j * BN, U.kvh, U.b);
                 }
             }
         }
@@ -627,7 +628,7 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
             const float vsc = kV16 ? v_scale[U.bkv] : 1.f;     // V = v_scale * (fp16 copy)
             const float inv_l = vsc / l;
             const bool valid = qi < Nq;
-            T *orow = o + ((long long)(U.b * Hq + hi) * Nq + qi) * D;
+            T *orow = o + U.b * os.b + hi * os.h + (long long)qi * os.n;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t v[32];
@@ -659,14 +660,22 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
 // ---- bf16 V -> fp16 V (per-KV-head power-of-two scale), for the kV16 kernel ----
 // Pass 1: per KV head, the largest finite |v| (as float bits: non-negative floats order like
 // their bit patterns, so an unsigned atomicMax finds it).
+// V rows are read through its strides (element offsets of head (b, g): b * vs.b + g * vs.h,
+// row n: + n * vs.n), D / 8 16-byte chunks per row.
+__device__ __forceinline__ const uint4 *fav_v_chunk(const uint16_t *v, FavStrides vs, int Hkv,
+                                                    long long head, long long i, int d8) {
+    const long long b = head / Hkv, g = head % Hkv, n = i / d8, c = i % d8;
+    return reinterpret_cast<const uint4 *>(v + b * vs.b + g * vs.h + n * vs.n + c * 8);
+}
+
 __global__ void __launch_bounds__(256)
-fav_vmax_kernel(const uint4 *__restrict__ v, unsigned *__restrict__ vmax_bits, long long per_head) {
+fav_vmax_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
+                unsigned *__restrict__ vmax_bits, long long per_head) {
     const long long head = blockIdx.y;
-    const uint4 *src = v + head * per_head;
     unsigned mx = 0;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_head;
          i += (long long)gridDim.x * blockDim.x) {
-        const uint4 w = src[i];
+        const uint4 w = *fav_v_chunk(v, vs, Hkv, head, i, d8);
         const uint32_t u[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -695,18 +704,17 @@ __device__ __forceinline__ int fav_v16_exponent(unsigned vmax_bits) {
 // 2^-31 of the head's maximum -- converts exactly; smaller values err by less than 2^(e-25).
 // Non-finite values stay non-finite.  Also stores v_scale = 2^e.
 __global__ void __launch_bounds__(256)
-fav_v16_kernel(const uint4 *__restrict__ v, uint4 *__restrict__ v16,
-               const unsigned *__restrict__ vmax_bits, float *__restrict__ v_scale,
-               long long per_head) {
+fav_v16_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
+               uint4 *__restrict__ v16, const unsigned *__restrict__ vmax_bits,
+               float *__restrict__ v_scale, long long per_head) {
     const long long head = blockIdx.y;
     const int e = fav_v16_exponent(vmax_bits[head]);
     if (blockIdx.x == 0 && threadIdx.x == 0) v_scale[head] = ldexpf(1.f, e);
     const float inv = ldexpf(1.f, -e);
-    const uint4 *src = v + head * per_head;
-    uint4 *dst = v16 + head * per_head;
+    uint4 *dst = v16 + head * per_head;        // contiguous [B, Hkv, Nkv, D]
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_head;
          i += (long long)gridDim.x * blockDim.x) {
-        const uint4 w = src[i];
+        const uint4 w = *fav_v_chunk(v, vs, Hkv, head, i, d8);
         const uint32_t u[4] = {w.x, w.y, w.z, w.w};
         uint32_t r[4];
 #pragma unroll
@@ -736,6 +744,7 @@ template <typename T, int D, bool kV16>
 fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
     using C = PrefillCfg<D>;
     const void *vsrc = a.v;
+    FavStrides vstr = a.vs;
     const float *v_scale = nullptr;
     if constexpr (kV16) {
         if (!workspace) return FAV_ERR_NO_MEMORY;
@@ -751,19 +760,20 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
         if (cudaMemsetAsync(vmax, 0, heads * sizeof(unsigned), stream) != cudaSuccess)
             return FAV_ERR_CUDA;
         fav_vmax_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(
-            static_cast<const uint4 *>(a.v), vmax, per_head);
+            static_cast<const uint16_t *>(a.v), a.vs, a.Hkv, D / 8, vmax, per_head);
         fav_v16_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(
-            static_cast<const uint4 *>(a.v), reinterpret_cast<uint4 *>(ws + L.v16), vmax, vsc,
-            per_head);
+            static_cast<const uint16_t *>(a.v), a.vs, a.Hkv, D / 8,
+            reinterpret_cast<uint4 *>(ws + L.v16), vmax, vsc, per_head);
         if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_v16_kernel", stream))
             return FAV_ERR_CUDA;
         vsrc = ws + L.v16;
+        vstr = fav_contiguous_strides(a.Hkv, a.Nkv, D);
         v_scale = vsc;
     }
     alignas(64) CUtensorMap tmQ, tmK, tmV;
-    fav_status st = fav_make_tmap_3d(&tmQ, a.q, D, a.Nq, a.B * a.Hq, BM);
-    if (st == FAV_OK) st = fav_make_tmap_3d(&tmK, a.k, D, a.Nkv, a.B * a.Hkv, BN);
-    if (st == FAV_OK) st = fav_make_tmap_3d(&tmV, vsrc, D, a.Nkv, a.B * a.Hkv, BN);
+    fav_status st = fav_make_tmap_4d(&tmQ, a.q, D, a.Nq, a.Hq, a.B, a.qs, BM);
+    if (st == FAV_OK) st = fav_make_tmap_4d(&tmK, a.k, D, a.Nkv, a.Hkv, a.B, a.ks, BN);
+    if (st == FAV_OK) st = fav_make_tmap_4d(&tmV, vsrc, D, a.Nkv, a.Hkv, a.B, vstr, BN);
     if (st != FAV_OK) return st;
     auto kern = fav_prefill_kernel<T, D, kV16>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
@@ -778,7 +788,7 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
     // persistent: one CTA per SM at most, each working through its share of the units
     const long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
     kern<<<(unsigned)blocks, kThreads, C::kSmemBytes, stream>>>(
-        tmQ, tmK, tmV, (T *)a.o, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
+        tmQ, tmK, tmV, (T *)a.o, a.os, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
         pair_heads, a.scale * kLog2e, a.causal, a.dev_status);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_kernel", stream))
         return FAV_ERR_CUDA;

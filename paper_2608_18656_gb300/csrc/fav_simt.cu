@@ -32,8 +32,9 @@ constexpr int kMaxD = 256;
 template <typename T>
 __global__ void __launch_bounds__(kWarps * 32)
 fav_simt_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restrict__ v,
-                T *__restrict__ o, float *__restrict__ lse, int Hq, int Hkv, int Nq, int Nkv,
-                int D, float scale, int causal, long long rows) {
+                T *__restrict__ o, FavStrides sq, FavStrides sk, FavStrides sv, FavStrides so,
+                float *__restrict__ lse, int Hq, int Hkv, int Nq, int Nkv, int D, float scale,
+                int causal, long long rows) {
     __shared__ float qs[kWarps][kMaxD];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long row = (long long)blockIdx.x * kWarps + warp;
@@ -43,9 +44,9 @@ fav_simt_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__res
     const int h = (int)(bh % Hq);
     const long long b = bh / Hq;
     const int g = h / (Hq / Hkv);
-    const T *qr = q + row * D;
-    const T *Kh = k + (b * Hkv + g) * (long long)Nkv * D;
-    const T *Vh = v + (b * Hkv + g) * (long long)Nkv * D;
+    const T *qr = q + b * sq.b + h * sq.h + (long long)i * sq.n;
+    const T *Kh = k + b * sk.b + g * sk.h;
+    const T *Vh = v + b * sv.b + g * sv.h;
     const int n = causal ? (Nkv - Nq + i + 1) : Nkv;
 
     for (int d = lane; d < D; d += 32) qs[warp][d] = ld(qr + d);
@@ -60,7 +61,7 @@ fav_simt_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__res
         const int j = j0 + lane;
         float s = -INFINITY;
         if (j < n) {
-            const T *kr = Kh + (long long)j * D;
+            const T *kr = Kh + (long long)j * sk.n;
             float dot = 0.f;
             for (int d = 0; d < D; ++d) dot = fmaf(qs[warp][d], ld(kr + d), dot);
             s = dot * scale;
@@ -81,7 +82,7 @@ fav_simt_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__res
         const int cnt = min(32, n - j0);
         for (int jj = 0; jj < cnt; ++jj) {
             const float pj = __shfl_sync(~0u, p, jj);
-            const T *vr = Vh + (long long)(j0 + jj) * D;
+            const T *vr = Vh + (long long)(j0 + jj) * sv.n;
 #pragma unroll
             for (int c = 0; c < kMaxD / 32; ++c) {
                 const int d = lane + 32 * c;
@@ -90,7 +91,7 @@ fav_simt_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__res
         }
     }
     const float inv = 1.f / l;
-    T *orow = o + row * D;
+    T *orow = o + b * so.b + h * so.h + (long long)i * so.n;
 #pragma unroll
     for (int c = 0; c < kMaxD / 32; ++c) {
         const int d = lane + 32 * c;
@@ -114,18 +115,19 @@ fav_status fav_launch_simt(const FavArgs &a, cudaStream_t s) {
     switch (a.dtype) {
     case FAV_F32:
         fav_simt_kernel<float><<<grid, block, 0, s>>>(
-            (const float *)a.q, (const float *)a.k, (const float *)a.v, (float *)a.o, a.lse,
-            a.Hq, a.Hkv, a.Nq, a.Nkv, a.D, a.scale, a.causal, rows);
+            (const float *)a.q, (const float *)a.k, (const float *)a.v, (float *)a.o, a.qs, a.ks,
+            a.vs, a.os, a.lse, a.Hq, a.Hkv, a.Nq, a.Nkv, a.D, a.scale, a.causal, rows);
         break;
     case FAV_F16:
         fav_simt_kernel<__half><<<grid, block, 0, s>>>(
-            (const __half *)a.q, (const __half *)a.k, (const __half *)a.v, (__half *)a.o, a.lse,
-            a.Hq, a.Hkv, a.Nq, a.Nkv, a.D, a.scale, a.causal, rows);
+            (const __half *)a.q, (const __half *)a.k, (const __half *)a.v, (__half *)a.o, a.qs,
+            a.ks, a.vs, a.os, a.lse, a.Hq, a.Hkv, a.Nq, a.Nkv, a.D, a.scale, a.causal, rows);
         break;
     case FAV_BF16:
         fav_simt_kernel<__nv_bfloat16><<<grid, block, 0, s>>>(
             (const __nv_bfloat16 *)a.q, (const __nv_bfloat16 *)a.k, (const __nv_bfloat16 *)a.v,
-            (__nv_bfloat16 *)a.o, a.lse, a.Hq, a.Hkv, a.Nq, a.Nkv, a.D, a.scale, a.causal, rows);
+            (__nv_bfloat16 *)a.o, a.qs, a.ks, a.vs, a.os, a.lse, a.Hq, a.Hkv, a.Nq, a.Nkv, a.D,
+            a.scale, a.causal, rows);
         break;
     }
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_simt_kernel", s)) return FAV_ERR_CUDA;
