@@ -167,6 +167,14 @@ FAV_API fav_status fav_set_decode_splits(int n);
 FAV_API int fav_last_decode_splits(void);
 
 /*
+ * fav_set_prefill_grid -- process-wide cap on the number of thread blocks of the persistent
+ * prefill kernel (0 = automatic: one per SM, at most one per query tile).  With a small cap
+ * each block works through many query tiles in turn, which tests use to exercise that path on
+ * small problems.  The results do not depend on the cap.  FAV_ERR_INVALID_ARG for n < 0.
+ */
+FAV_API fav_status fav_set_prefill_grid(int n);
+
+/*
  * fav_decode_noalloc -- the decode path (split-KV decode kernel + log-sum-exp combine) with no
  * device allocation at all.  The paper has no counterpart: this entry point exists for callers
  * that cannot let a library allocate device memory -- a server whose own pool reserves all

@@ -8,7 +8,7 @@ import ctypes
 import os
 
 __all__ = ["forward", "forward_host", "Strides", "set_path", "last_path", "set_decode_splits",
-           "last_decode_splits", "device_status", "release_workspace", "library_path",
+           "last_decode_splits", "set_prefill_grid", "device_status", "release_workspace", "library_path",
            "FavError", "F32", "F16", "BF16", "PATH_AUTO", "PATH_SIMT", "PATH_DECODE",
            "PATH_PREFILL"]
 
@@ -71,6 +71,8 @@ def lib():
         L.fav_set_decode_splits.restype = i
         L.fav_last_decode_splits.argtypes = []
         L.fav_last_decode_splits.restype = i
+        L.fav_set_prefill_grid.argtypes = [i]
+        L.fav_set_prefill_grid.restype = i
         _lib = L
     return _lib
 
@@ -166,6 +168,11 @@ def set_decode_splits(n):
 
 def last_decode_splits():
     return lib().fav_last_decode_splits()
+
+
+def set_prefill_grid(n):
+    """Cap on the persistent prefill kernel's thread blocks (0 = one per SM)."""
+    _check(lib().fav_set_prefill_grid(int(n)))
 
 
 def device_status():

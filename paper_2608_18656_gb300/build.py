@@ -12,7 +12,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libfav.so")
-SOURCES = ["fav_api.cu", "fav_simt.cu", "fav_decode.cu", "fav_prefill.cu", "fav_noalloc.cu"]
+SOURCES = ["fav_api.cu", "fav_simt.cu", "fav_decode.cu", "fav_prefill.cu", "fav_prefill_pair.cu",
+           "fav_v16.cu", "fav_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

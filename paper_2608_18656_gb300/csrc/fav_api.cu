@@ -44,6 +44,7 @@ std::atomic<int> g_path{FAV_PATH_AUTO};
 std::atomic<int> g_last_path{FAV_PATH_AUTO};
 std::atomic<int> g_splits{0};
 std::atomic<int> g_last_splits{0};
+std::atomic<int> g_prefill_grid{0};
 
 fav_status device_state(DeviceState **out) {
     int dev = 0;
@@ -140,6 +141,7 @@ fav_status forward_impl(const FavArgs &in, cudaStream_t stream) {
     FavArgs a = in;
     a.dev_status = ds->status;
     a.num_sms = ds->num_sms;
+    a.prefill_grid = g_prefill_grid.load();
     const fav_path path = choose_path(a);
     if (path == FAV_PATH_AUTO) return FAV_ERR_UNSUPPORTED;
     cudaGetLastError();   // a stale error from elsewhere must not be reported as ours
@@ -212,8 +214,7 @@ bool fav_debug_sync(const char *what, cudaStream_t s) {
     return e != cudaSuccess;
 }
 
-fav_status fav_make_tmap_4d(void *tmap, const void *base, int D, int rows, int heads, int batch,
-                            FavStrides st, int box_rows) {
+static PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
     static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     static std::once_flag once;
     std::call_once(once, [] {
@@ -224,6 +225,12 @@ fav_status fav_make_tmap_4d(void *tmap, const void *base, int D, int rows, int h
             q == cudaDriverEntryPointSuccess)
             encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     });
+    return encode;
+}
+
+fav_status fav_make_tmap_4d(void *tmap, const void *base, int D, int rows, int heads, int batch,
+                            FavStrides st, int box_rows) {
+    const PFN_cuTensorMapEncodeTiled_v12000 encode = tmap_encoder();
     if (!encode) return FAV_ERR_CUDA;
     const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)heads,
                                 (cuuint64_t)batch};
@@ -237,6 +244,32 @@ fav_status fav_make_tmap_4d(void *tmap, const void *base, int D, int rows, int h
     const cuuint32_t box[4] = {64, (cuuint32_t)box_rows, 1, 1};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     CUresult r = encode(reinterpret_cast<CUtensorMap *>(tmap), CU_TENSOR_MAP_DATA_TYPE_UINT16, 4,
+                        const_cast<void *>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? FAV_OK : FAV_ERR_CUDA;
+}
+
+// 5-D view (64 elements, rows, D / 64 column blocks, heads, batch) of a [B, H, N, D] tensor: a
+// box of box_rows rows spans all D columns in ONE copy instruction and lands in shared memory
+// as D / 64 consecutive 64-column blocks of box_rows x 128 bytes (128-byte swizzle) -- the same
+// layout as D / 64 separate 64-column boxes.  (A TMA engine's throughput per issuing thread is
+// bounded per instruction, so one copy per tile instead of two matters for D = 128.)
+fav_status fav_make_tmap_tiles(void *tmap, const void *base, int D, int rows, int heads,
+                               int batch, FavStrides st, int box_rows) {
+    const PFN_cuTensorMapEncodeTiled_v12000 encode = tmap_encoder();
+    if (!encode) return FAV_ERR_CUDA;
+    const int blocks = D / 64;
+    const cuuint64_t dims[5] = {64, (cuuint64_t)rows, (cuuint64_t)blocks, (cuuint64_t)heads,
+                                (cuuint64_t)batch};
+    auto bstride = [](long long e, long long fallback) {
+        return (cuuint64_t)((e > 0 ? e : fallback) * 2);
+    };
+    const cuuint64_t strides[4] = {bstride(st.n, D), 128, bstride(st.h, (long long)rows * D),
+                                   bstride(st.b, (long long)heads * rows * D)};
+    const cuuint32_t box[5] = {64, (cuuint32_t)box_rows, (cuuint32_t)blocks, 1, 1};
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    CUresult r = encode(reinterpret_cast<CUtensorMap *>(tmap), CU_TENSOR_MAP_DATA_TYPE_UINT16, 5,
                         const_cast<void *>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -430,5 +463,11 @@ fav_status fav_set_decode_splits(int n) {
 }
 
 int fav_last_decode_splits(void) { return g_last_splits.load(); }
+
+fav_status fav_set_prefill_grid(int n) {
+    if (n < 0) return FAV_ERR_INVALID_ARG;
+    g_prefill_grid.store(n);
+    return FAV_OK;
+}
 
 }  // extern "C"

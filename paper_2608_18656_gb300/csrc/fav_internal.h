@@ -21,6 +21,7 @@ struct FavArgs {
     fav_dtype dtype;
     int *dev_status;   // device word set by bounded waits that gave up
     int num_sms;
+    int prefill_grid = 0;   // cap on the persistent prefill grid (0 = one CTA per SM)
 };
 
 // Generic CUDA-core kernel (fav_simt.cu).
@@ -39,6 +40,15 @@ bool fav_prefill_supported(const FavArgs &a);
 // Device workspace the prefill launch needs (0 for fp16; bf16: the fp16 copy of V and its
 // per-head scales), and the launch itself with that workspace.
 size_t fav_prefill_workspace_bytes(const FavArgs &a);
+// bf16 V -> fp16 V with a power-of-two scale per KV head (fav_v16.cu), for the prefill
+// kernels: workspace size, and the conversion (two kernels on `stream`), which returns the
+// fp16 copy (contiguous [B, Hkv, Nkv, D], its strides) and the per-head scales 2^e.
+size_t fav_v16_workspace_bytes(const FavArgs &a);
+fav_status fav_v16_convert(const FavArgs &a, void *workspace, cudaStream_t stream,
+                           const void **v16, FavStrides *v16_strides, const float **v_scale);
+// The two prefill kernel designs (fav_prefill.cu: D = 128; fav_prefill_pair.cu: D = 64).
+fav_status fav_launch_prefill_split(const FavArgs &a, void *workspace, cudaStream_t s);
+fav_status fav_launch_prefill_pair(const FavArgs &a, void *workspace, cudaStream_t s);
 fav_status fav_launch_prefill(const FavArgs &a, void *workspace, cudaStream_t s);
 
 // With FAV_DEBUG_SYNC=1 in the environment: synchronise `s` after a launch and report a
@@ -64,3 +74,7 @@ inline FavStrides fav_contiguous_strides(int H, int N, int D) {
 // 128-byte swizzle, zero fill out of bounds.  Coordinates (x, row, head, batch).
 fav_status fav_make_tmap_4d(void *tmap /* CUtensorMap* */, const void *base, int D, int rows,
                             int heads, int batch, FavStrides st, int box_rows);
+// The same tensor as a 5-D view whose box of box_rows rows covers all D columns in one TMA
+// copy (D / 64 blocks of 64 columns, each box_rows x 128 bytes, 128-byte swizzle).
+fav_status fav_make_tmap_tiles(void *tmap /* CUtensorMap* */, const void *base, int D, int rows,
+                               int heads, int batch, FavStrides st, int box_rows);

@@ -1,41 +1,47 @@
-// fav_prefill.cu -- prefill attention on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
+// fav_prefill.cu -- prefill attention for D = 128 on the 5th-generation tensor cores
+// (tcgen05 + TMEM + TMA): one query tile per unit of work, the softmax split over the keys.
 //
 // Method (paper, Algorithm "FlashAttention-V for VL > D" and its description): the query
 // rows of a block stay on chip for the whole sweep over key/value blocks; for every key block
 // the scores are computed, the running maximum / sum / output accumulator of the online
 // softmax are updated (rescale by exp(M_old - M), weights exp(S - M)), and after the last
 // block the accumulator is normalised.  Heads sharing a K/V head read the same K/V tiles
-// (GQA reuse), and several heads are processed by one unit of work (the paper's inter-head
-// parallelism).  On this GPU that becomes:
-//   * a unit is two 128-row query tiles that read the same K/V head: the same query tile of
-//     two heads of one GQA group (even group sizes), or two consecutive query tiles of one
-//     head.  The kernel is persistent (one CTA per SM at most); CTA c works through units
-//     c, 2P-1-c, 2P+c, ... of the units sorted by decreasing causal work, loading the next
-//     unit's Q tiles (TMA, 128-byte swizzle) during the current unit's tail;
-//   * 128-key K and V tiles are streamed by TMA through a ring of shared-memory stages and
-//     serve both query tiles;
-//   * S_i = Q_i K^T (M = 128, N = 128, K = D) and O_i += P_i V (M = 128, N = D, K = 128) are
-//     bursts of tcgen05.mma issued by one elected lane of a converged warp, accumulating in
-//     tensor memory (TMEM), with P_i read from TMEM;
-//   * one softmax warpgroup per query tile, one thread per query row (= TMEM lane): tcgen05.ld
-//     of its scores, mask, row maximum, exp2 in the log2 domain, row sum, fp16 weights stored
-//     with tcgen05.st.
-// D = 128: TMEM holds S0 | S1 | O0 | O1 and P_i overwrites the first half of S_i, so S_i(j+1)
-// can only follow P_i(j).V; the MMA warp alternates [P_0(j).V, S_0(j+1)], [P_1(j).V, S_1(j+1)]
-// and each softmax runs while the tensor core works on the other tile.  D = 64: the weights
-// have columns of their own (S0 | S1 | P0 | P1 | O0 | O1), S_i(j+1) is issued as soon as the
-// softmax has read S_i(j), and the two tiles' softmaxes run back to back, half a period apart.
-// The running maximum is updated lazily: O and l are rescaled only when the maximum grows by
-// more than 2^4 (log2 domain); the weights are stored as p * 2^11 (below 2^15, inside fp16's
-// range).  The final O / l uses the same maximum as every weight, so the result is unchanged.
+// (GQA reuse: neighbouring CTAs work on the heads of one group at the same time, so the tiles
+// come from L2).  On this GPU that becomes:
+//   * a unit is one 128-row query tile; the kernel is persistent (one CTA per SM at most) and
+//     CTA c works through units c, 2P-1-c, 2P+c, ... of the units sorted by decreasing causal
+//     work, with the next unit's Q tile loaded (TMA, 128-byte swizzle) into a second buffer;
+//   * 128-key K and V tiles are streamed by TMA (one copy instruction per tile) through rings
+//     of shared-memory stages;
+//   * S = Q K^T (M = 128, N = 128, K = 128) goes to one of two TMEM score buffers, so the
+//     tensor core computes the scores of key tile j+1 while the softmax works on tile j;
+//   * the softmax of a tile is split over the keys: split s (of two) owns keys
+//     [64 s, 64 s + 64) of every tile and keeps its own running maximum, sum and output
+//     accumulator O_s (128 TMEM columns) -- the online softmax applied to each key subset
+//     separately, as in the split-KV decode.  O_s += P_s V_s is a burst of tcgen05.mma with
+//     the weights P_s read from TMEM.  The splits are merged once per unit:
+//     O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, M = max_s m_s.
+//     The point of the split: a tile's softmax runs on eight warps (two per scheduler) with no
+//     exchange between them, and takes about as long as the tile's MMAs.
+//   * the merged O tile is written into the unit's (by then free) Q buffer and stored with
+//     one TMA tensor store.
+// TMEM (512 columns): score buffers 0 | 1 (128 columns each; the fp16 weights of split s
+// overwrite the first half of its own score columns), then O_0 | O_1.
+// The running maximum is updated lazily: O_s and l_s are rescaled only when the maximum grows
+// by more than 2^4 (log2 domain); the weights are stored as p * 2^11 (below 2^15, inside
+// fp16's range).  O_s / l_s keeps the same maximum as its weights, so the result is unchanged.
 //
-// Warp roles (320 threads): warps 0-3 softmax of tile 0, warps 4-7 softmax of tile 1
-// (TMEM lane quarter = warp % 4); warp 8 = TMEM owner + MMA issuer (the whole warp, one
-// elected lane issuing each burst and committing the barrier arrivals inside the same asm
-// block); warp 9 = TMA producer.  The issuing lane blocks while the tensor pipe is busy, and a
-// wait on an mbarrier costs ~80 cycles of latency even when the phase is already complete; so
-// the warp tests the barriers it will need next *before* a burst of MMAs where it can, and
-// only waits for real on the ones that were not complete.
+// Warp roles (384 threads): warps 0-7 softmax (TMEM lane quarter = warp % 4, key split =
+// warp / 4; one thread per query row and split); warp 8 = TMEM owner + MMA issuer (the whole
+// warp, one elected lane issuing each burst and committing the barrier arrivals inside the
+// same asm block); warp 9 = Q/K producer, warp 10 = V producer (two issuing warps keep more TMA
+// copies in flight than one); warp 11 = O stores.
+//
+// Issue order of the tensor core, per CTA over the global sequence G of key tiles (all units):
+//   S(0), S(1), P(0).V, S(2), P(1).V, S(3), ...    S(G) into score buffer G % 2
+// S(G + 2) overwrites the weights of tile G, so it follows P(G).V in the same (in-order) pipe.
+// (For D = 64 the two-tile kernel of fav_prefill_pair.cu is faster: its products are short
+// and two query tiles sharing each K/V tile keep the softmax warps busier.)
 #include <cuda.h>
 #include <math.h>
 
@@ -58,8 +64,6 @@ namespace {
 
 constexpr int BM = 128;          // query rows per tile (= TMEM lanes)
 constexpr int BN = 128;          // keys per tile
-constexpr int kThreads = 320;
-constexpr int kMmaWarp = 8, kLoadWarp = 9;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleThreshold = 4.0f;   // log2 units: rescale when max grows by > 2^4
@@ -68,14 +72,6 @@ constexpr float kRescaleThreshold = 4.0f;   // log2 units: rescale when max grow
 // 2^-25 of the reference stay fp16 normals.  O / l is unchanged (l carries the same factor);
 // the LSE subtracts kPShift.
 constexpr float kPShift = 11.0f;
-
-// 2^x for a pair of weights with ex2 on the special-function unit.  (Computing a share of them
-// with a polynomial on the FMA pipe was measured slower on this GPU: the softmax is bound by
-// issue slots and latency, not by the ex2 rate.)
-template <int kPair>
-__device__ __forceinline__ float2 exp2_pair(float2 x) {
-    return make_float2(fav::fast_exp2(x.x), fav::fast_exp2(x.y));
-}
 
 // Calls f(std::integral_constant-like index) for kI = 0 .. kN-1, each a compile-time constant.
 template <int kI, int kN, typename F>
@@ -99,76 +95,86 @@ template <> struct IsBF16<__nv_bfloat16> { static constexpr bool value = true; }
 // than the others.
 
 template <int D> struct PrefillCfg {
-    static constexpr int kStages = (D == 128) ? 2 : 3;      // K/V ring depth
-    static constexpr int kBoxes = D / 64;
-    static constexpr int kQBytes = BM * D * 2;               // one Q tile
+    static_assert(D == 128, "the key-split kernel serves D = 128");
+    static constexpr int kSplits = 2;                        // key splits per tile
+    static constexpr int kSplitKeys = BN / kSplits;          // keys per split and tile
+    static constexpr int kSoftWarps = 4 * kSplits;
+    static constexpr int kMmaWarp = kSoftWarps;
+    static constexpr int kLoadKWarp = kSoftWarps + 1;        // Q and K
+    static constexpr int kLoadVWarp = kSoftWarps + 2;
+    static constexpr int kStoreWarp = kSoftWarps + 3;        // O tiles (TMA store)
+    static constexpr int kThreads = 32 * (kSoftWarps + 4);
+    static constexpr int kKStages = 2;                       // K ring depth
+    static constexpr int kVStages = 2;                       // V ring depth
+    static constexpr int kQBytes = BM * D * 2;               // one Q tile (or one O tile)
     static constexpr int kKVBytes = BN * D * 2;              // one K or V tile
+    static constexpr int kUnitTab = 256;                     // units precomputed per CTA
     // shared-memory map (offsets from the 1024-aligned base)
-    static constexpr int kOffQ = 0;                          // Q tile 0, Q tile 1
+    static constexpr int kOffQ = 0;                          // Q buffers 0, 1 (O staging)
     static constexpr int kOffK = kOffQ + 2 * kQBytes;
-    static constexpr int kOffV = kOffK + kStages * kKVBytes;
-    static constexpr int kOffBar = kOffV + kStages * kKVBytes;
-    static constexpr int kNumBars = 2 + 1 + 4 * kStages + 2 + 2 + 2 + 2 + 2;
+    static constexpr int kOffV = kOffK + kKStages * kKVBytes;
+    static constexpr int kOffXch = kOffV + kVStages * kKVBytes;   // (m, l) [2][4][splits][32]
+    static constexpr int kXchBytes = 2 * 4 * kSplits * 32 * 8;
+    static constexpr int kOffUnits = kOffXch + kXchBytes;         // int[kUnitTab][8]
+    static constexpr int kOffBar = kOffUnits + kUnitTab * 32;
+    static constexpr int kNumBars = 2 + 2 + 2 * kKStages + 2 * kVStages + 2 + 2 + 2 + 8 + 2;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
     static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
-    // TMEM columns.  D = 128: S0 | S1 | O0 | O1, and P_i (fp16, two weights per column)
-    // aliases the first 64 columns of S_i.  D = 64 (kSepP): S0 | S1 | P0 | P1 | O0 | O1, the
-    // weights have columns of their own, so the next scores of a tile can be computed while its
-    // softmax still works on the current ones.
-    static constexpr bool kSepP = (D == 64);
     static constexpr uint32_t kTmemCols = 512;
-    static __host__ __device__ constexpr uint32_t colS(int i) { return i ? 128u : 0u; }
-    static __host__ __device__ constexpr uint32_t colP(int i) { return kSepP ? 256u + 64u * i : colS(i); }
-    static __host__ __device__ constexpr uint32_t colO(int i) {
-        return kSepP ? 384u + 64u * i : 256u + (i ? D : 0);
-    }
-    static_assert(kSepP ? 384 + 2 * D <= 512 : 256 + 2 * D <= 512, "TMEM budget");
+    static __host__ __device__ constexpr uint32_t colS(int buf) { return buf ? 128u : 0u; }
+    static constexpr uint32_t kColO = 256;                   // O_s at kColO + s * D
+    static_assert(256 + kSplits * D == 512, "TMEM budget");
+    static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 };
 
 // bf16 I/O (kV16): Q, K and O are bf16; V has been converted to fp16 (tmV, scaled per KV head
 // by v_scale^-1, a power of two) so that P.V runs with fp16 weights, and the epilogue multiplies
 // O back by v_scale.  fp16 I/O: tmV is V itself.
 template <typename T, int D, bool kV16>
-__global__ void __launch_bounds__(kThreads, 1)
-fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   const __grid_constant__ CUtensorMap tmV, T *__restrict__ o, FavStrides os,
-                   float *__restrict__ lse, const float *__restrict__ v_scale, int B, int Hq,
-                   int Hkv, int Nq, int Nkv, int n_qtiles, int pair_heads, float scale_log2,
-                   int causal, int *status) {
+__global__ void __launch_bounds__(PrefillCfg<D>::kThreads, 1)
+fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
+                         const __grid_constant__ CUtensorMap tmK,
+                         const __grid_constant__ CUtensorMap tmV,
+                         const __grid_constant__ CUtensorMap tmO, float *__restrict__ lse, const float *__restrict__ v_scale, int B, int Hq,
+                   int Hkv, int Nq, int Nkv, int n_qtiles, float scale_log2, int causal,
+                   int *status) {
     using C = PrefillCfg<D>;
     using TP = __half;    // type of the weights P and of V in shared memory (P.V MMA)
-    constexpr int S = C::kStages;
+    constexpr int KS = C::kKStages, VS = C::kVStages, NS = C::kSplits, SK = C::kSplitKeys;
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment in the shared window (the 128-byte swizzle atom of TMA and MMA)
     const uint32_t raw_u32 = fav::smem_u32(smem_raw);
     uint8_t *smem = smem_raw + ((1024u - (raw_u32 & 1023u)) & 1023u);
     const uint32_t sbase = fav::smem_u32(smem);
-    const uint32_t sK = sbase + C::kOffK, sV = sbase + C::kOffV;
+    const uint32_t sQ = sbase + C::kOffQ, sK = sbase + C::kOffK, sV = sbase + C::kOffV;
     const uint32_t bar0 = sbase + C::kOffBar;
-    const uint32_t q_full = bar0;                 // [2], one per query tile
-    const uint32_t q_empty = q_full + 16;         // Q buffers free (last S MMA of a unit done)
-    const uint32_t k_full = q_empty + 8, k_empty = k_full + 8 * S;
-    const uint32_t v_full = k_empty + 8 * S, v_empty = v_full + 8 * S;
-    const uint32_t s_full = v_empty + 8 * S;      // [2], one per query tile
-    const uint32_t p_full = s_full + 16;          // [2]
-    const uint32_t o_done = p_full + 16;          // [2]
-    const uint32_t s_free = o_done + 16;          // [2] (kSepP) the softmax has read S_i
-    const uint32_t p_free = s_free + 16;          // [2] (kSepP) P_i.V has completed
+    const uint32_t q_full = bar0;                 // [2] per Q buffer
+    const uint32_t q_empty = q_full + 16;         // [2] the buffer's last S read and O stored
+    const uint32_t k_full = q_empty + 16, k_empty = k_full + 8 * KS;
+    const uint32_t v_full = k_empty + 8 * KS, v_empty = v_full + 8 * VS;
+    const uint32_t s_full = v_empty + 8 * VS;     // [2] per score buffer
+    const uint32_t p_full = s_full + 16;          // [2] per score buffer (weights stored)
+    const uint32_t pv_done = p_full + 16;         // P(G).V completed, once per key tile
+    const uint32_t o_done = pv_done + 8;          // a unit's last P.V completed, once per unit
+    const uint32_t xch_bar = o_done + 8;          // [2][4] split (m, l) exchange per quarter
+    const uint32_t o_staged = xch_bar + 64;       // [2] O tile written into Q buffer k % 2
+    float2 *xch = reinterpret_cast<float2 *>(smem + C::kOffXch);
+    int *utab = reinterpret_cast<int *>(smem + C::kOffUnits);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffTmemSlot);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int G = Hq / Hkv;
     const int off = Nkv - Nq;                                   // bottom-right causal offset
+    const int BH = B * Hq;
 
-    // ---- work units: two query tiles that read the same K/V head, heaviest causal first ----
-    // Unit u: the same query tile of two heads of one GQA group (even group sizes), or two
-    // consecutive query tiles of one head.  The CTA takes units c, 2P-1-c, 2P+c, 4P-1-c, ...
-    // (P CTAs, "snake" order): with the units sorted by decreasing work, this evens out the
-    // sums per CTA.
+    // ---- work units: one query tile each, heaviest causal first ----
+    // Unit u: query tile t = n_qtiles - 1 - u / (B * Hq) of head (b, h) = u % (B * Hq), so the
+    // heads of one GQA group (consecutive h) run side by side.  The CTA takes units c, 2P-1-c,
+    // 2P+c, 4P-1-c, ... (P CTAs, "snake" order), which evens out the work per CTA.
     struct Unit {
-        int b, h[2], t[2], n_kv_tiles[2], n_kv, kvh, bkv;
+        int b, h, t, n_kv, kvh;
     };
-    const int n_units = pair_heads ? n_qtiles * B * (Hq / 2) : ((n_qtiles + 1) / 2) * B * Hq;
+    const int n_units = n_qtiles * BH;
     auto unit_at = [&](int k) {   // the k-th unit of this CTA, or -1
         const int P = gridDim.x, c = blockIdx.x;
         const int u = k * P + ((k & 1) ? (P - 1 - c) : c);
@@ -176,64 +182,62 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     };
     auto make_unit = [&](int u) {
         Unit U;
-        if (pair_heads) {
-            const int units = B * (Hq / 2);
-            const int r = u % units;
-            U.t[0] = U.t[1] = n_qtiles - 1 - u / units;
-            U.b = r / (Hq / 2);
-            U.h[0] = 2 * (r % (Hq / 2));
-            U.h[1] = U.h[0] + 1;
-        } else {
-            const int BH = B * Hq;
-            const int n_pairs = (n_qtiles + 1) / 2;
-            const int bh = u % BH;
-            const int pr = n_pairs - 1 - u / BH;
-            U.b = bh / Hq;
-            U.h[0] = U.h[1] = bh % Hq;
-            U.t[0] = 2 * pr;
-            U.t[1] = 2 * pr + 1;
-        }
-        U.kvh = U.h[0] / G;
-        U.bkv = U.b * Hkv + U.kvh;
-#pragma unroll
-        for (int i = 0; i < 2; ++i) {
-            if (U.t[i] >= n_qtiles) {
-                U.n_kv_tiles[i] = 0;
-            } else {
-                const int kv_end = causal ? min(Nkv, U.t[i] * BM + BM + off) : Nkv;
-                U.n_kv_tiles[i] = (kv_end + BN - 1) / BN;
-            }
-        }
-        U.n_kv = max(U.n_kv_tiles[0], U.n_kv_tiles[1]);
+        const int bh = u % BH;
+        U.t = n_qtiles - 1 - u / BH;
+        U.b = bh / Hq;
+        U.h = bh % Hq;
+        U.kvh = U.h / G;
+        const int kv_end = causal ? min(Nkv, U.t * BM + BM + off) : Nkv;
+        U.n_kv = (kv_end + BN - 1) / BN;
         return U;
     };
+    // The CTA's first kUnitTab units are computed once, in parallel, into shared memory (the
+    // integer divisions would otherwise sit on the critical path at every unit switch).
+    auto unit = [&](int k) {
+        if (k < C::kUnitTab) {
+            const int *e = utab + 8 * k;
+            Unit U;
+            U.b = e[0]; U.h = e[1]; U.t = e[2]; U.n_kv = e[3]; U.kvh = e[4];
+            return U;
+        }
+        return make_unit(unit_at(k));
+    };
+    for (int k = threadIdx.x; k < C::kUnitTab; k += blockDim.x) {
+        const int u = unit_at(k);
+        if (u < 0) break;
+        const Unit U = make_unit(u);
+        int *e = utab + 8 * k;
+        e[0] = U.b; e[1] = U.h; e[2] = U.t; e[3] = U.n_kv; e[4] = U.kvh;
+    }
 
-    if (warp == kLoadWarp && lane == 0) {
+    if (warp == C::kLoadKWarp && lane == 0) {
         (void)FAV_CHECK((sbase & 1023u) == 0, status);
         (void)FAV_CHECK((sbase - raw_u32) + C::kOffTmemSlot + 4 <= fav::dynamic_smem_bytes(), status);
-        fav::mbar_init(q_full, 1);
-        fav::mbar_init(q_full + 8, 1);
-        fav::mbar_init(q_empty, 1);
-        for (int s = 0; s < S; ++s) {
+        for (int i = 0; i < 2; ++i) {
+            fav::mbar_init(q_full + 8 * i, 1);
+            fav::mbar_init(q_empty + 8 * i, 2);          // last S commit + O store read
+            fav::mbar_init(o_staged + 8 * i, C::kSoftWarps * 32);
+            fav::mbar_init(s_full + 8 * i, 1);
+            fav::mbar_init(p_full + 8 * i, C::kSoftWarps);
+        }
+        for (int s = 0; s < KS; ++s) {
             fav::mbar_init(k_full + 8 * s, 1);
             fav::mbar_init(k_empty + 8 * s, 1);
+        }
+        for (int s = 0; s < VS; ++s) {
             fav::mbar_init(v_full + 8 * s, 1);
             fav::mbar_init(v_empty + 8 * s, 1);
         }
-        for (int i = 0; i < 2; ++i) {
-            fav::mbar_init(s_full + 8 * i, 1);
-            fav::mbar_init(p_full + 8 * i, 4);
-            fav::mbar_init(o_done + 8 * i, 1);
-            fav::mbar_init(s_free + 8 * i, 4);
-            fav::mbar_init(p_free + 8 * i, 1);
-        }
+        fav::mbar_init(pv_done, 1);
+        fav::mbar_init(o_done, 1);
+        for (int i = 0; i < 8; ++i) fav::mbar_init(xch_bar + 8 * i, NS * 32);
         fav::mbar_fence_init();
     }
 #ifdef FAV_TIMING
     __shared__ long long t_ref;
     if (threadIdx.x == 0) t_ref = clock64();
 #endif
-    if (warp == kMmaWarp) {
+    if (warp == C::kMmaWarp) {
         fav::tc::tmem_alloc(fav::smem_u32(tmem_slot), C::kTmemCols);
         fav::tc::tmem_relinquish();
     }
@@ -243,352 +247,357 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     const uint32_t tmem = *tmem_slot;
     (void)FAV_CHECK((tmem & 0xFFFFu) + C::kTmemCols <= 512u && (tmem >> 16) == 0u, status);
 
-    // Barrier phases run on across units: K/V stages follow one sequence g of key tiles
-    // (stage g % S, parity (g / S) & 1) on both sides; s_full / p_full of tile i complete once
-    // per key tile of i, o_done once per unit in which tile i has work, q_full once per unit.
-    if (warp == kLoadWarp) {
-        // ---------------- TMA producer ----------------
+    // Barrier phases run on across units: key tile G of the CTA's sequence uses K stage G % KS
+    // (parity (G / KS) & 1), V stage G % VS, score buffer G % 2 (s_full / p_full parity
+    // (G / 2) & 1) and completes pv_done phase G; unit k uses Q buffer k % 2 (parity
+    // (k / 2) & 1) and exchange slot k % 2, and completes o_done phase k.
+    if (warp == C::kLoadKWarp) {
+        // ---------------- TMA producer: Q tiles and K tiles ----------------
         if (lane == 0) {
             fav::tma_prefetch_desc(&tmQ);
             fav::tma_prefetch_desc(&tmK);
+            int g = 0;
+            bool ok = true;
+            for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
+                const Unit U = unit(k);
+                const int qb = k & 1;
+                // Q buffer qb was last read by unit k - 2's S MMAs
+                if (k >= 2 && !fav::mbar_wait(q_empty + 8 * qb, ((k >> 1) - 1) & 1, status)) break;
+                fav::mbar_arrive_expect_tx(q_full + 8 * qb, C::kQBytes);
+                fav::tma_load_5d(sQ + qb * C::kQBytes, &tmQ, q_full + 8 * qb, 0, U.t * BM, 0, U.h, U.b);
+                for (int j = 0; j < U.n_kv; ++j, ++g) {
+                    const int st = g % KS;
+                    if (g >= KS && !fav::mbar_wait(k_empty + 8 * st, ((g / KS) - 1) & 1, status)) {
+                        ok = false;
+                        break;
+                    }
+                    fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
+                    fav::tma_load_5d(sK + st * C::kKVBytes, &tmK, k_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
+                }
+            }
+        }
+    } else if (warp == C::kLoadVWarp) {
+        // ---------------- TMA producer: V tiles ----------------
+        if (lane == 0) {
             fav::tma_prefetch_desc(&tmV);
             int g = 0;
             bool ok = true;
             for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
-                const Unit U = make_unit(u);
-                // the Q buffers are free once the previous unit's last S MMA has completed; both
-                // tiles are loaded (a tile beyond the sequence reads the zero fill)
-                if (k > 0 && !fav::mbar_wait(q_empty, (k - 1) & 1, status)) break;
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    fav::mbar_arrive_expect_tx(q_full + 8 * i, C::kQBytes);
-#pragma unroll
-                    for (int bx = 0; bx < C::kBoxes; ++bx)
-                        fav::tma_load_4d(sbase + C::kOffQ + i * C::kQBytes + bx * BM * 128, &tmQ,
-                                         q_full + 8 * i, bx * 64, U.t[i] * BM, U.h[i], U.b);
-                }
-                // Each stage has its own empty barriers (one commit per use, waited in order).
+                const Unit U = unit(k);
                 for (int j = 0; j < U.n_kv; ++j, ++g) {
-                    const int st = g % S;
-                    const uint32_t ph = ((g / S) + 1) & 1;   // parity of the previous use's phase
-                    if (g >= S && !fav::mbar_wait(k_empty + 8 * st, ph, status)) { ok = false; break; }
-                    fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
-#pragma unroll
-                    for (int bx = 0; bx < C::kBoxes; ++bx)
-                        fav::tma_load_4d(sK + st * C::kKVBytes + bx * BN * 128, &tmK, k_full + 8 * st,
-                                         bx * 64, j * BN, U.kvh, U.b);
-                    if (g >= S && !fav::mbar_wait(v_empty + 8 * st, ph, status)) { ok = false; break; }
+                    const int st = g % VS;
+                    if (g >= VS && !fav::mbar_wait(v_empty + 8 * st, ((g / VS) - 1) & 1, status)) {
+                        ok = false;
+                        break;
+                    }
                     fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
-#pragma unroll
-                    for (int bx = 0; bx < C::kBoxes; ++bx)
-                        fav::tma_load_4d(sV + st * C::kKVBytes + bx * BN * 128, &tmV, v_full + 8 * st,
-                                         bx * 64, j * BN, U.kvh, U.b);
+                    fav::tma_load_5d(sV + st * C::kKVBytes, &tmV, v_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
                 }
             }
         }
-    } else if (warp == kMmaWarp) {
+    } else if (warp == C::kStoreWarp) {
+        // ---------------- O tiles: one TMA store per unit from its (free) Q buffer ----------------
+        if (lane == 0) {
+            fav::tma_prefetch_desc(&tmO);
+            for (int k = 0, u; (u = unit_at(k)) >= 0; ++k) {
+                const Unit U = unit(k);
+                const int qb = k & 1;
+                if (!fav::mbar_wait(o_staged + 8 * qb, (k >> 1) & 1, status)) break;
+                fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.t * BM, 0, U.h, U.b);
+                fav::bulk_commit_group();
+                fav::bulk_wait_read_all();         // the buffer may take the next Q tile
+                fav::mbar_arrive(q_empty + 8 * qb);
+            }
+            fav::bulk_wait_all();
+        }
+    } else if (warp == C::kMmaWarp) {
         // ---------------- MMA issuer: the whole warp, converged; one elected lane issues ----------------
         constexpr bool bf = IsBF16<T>::value;
         constexpr uint32_t idesc_qk = fav::tc::idesc_f16(BM, BN, bf, false);
         constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, false, true);      // fp16 P, V
         // Base descriptors are built once; a tile only adds its byte offset (>> 4) to the
         // start-address field, which cannot carry out of its 14 bits (addresses < 256 KB).
-        const uint64_t dq0 = fav::tc::sdesc_sw128(sbase + C::kOffQ, 16, 1024);
+        const uint64_t dq0 = fav::tc::sdesc_sw128(sQ, 16, 1024);
         const uint64_t dk0 = fav::tc::sdesc_sw128(sK, 16, 1024);
         const uint64_t dv0 = fav::tc::sdesc_sw128(sV, BN * 128, 1024);
-        // S_i = Q_i K^T (K in ring stage st): D/16 k-steps over the 64-column boxes of Q_i and
-        // K; the burst ends with commits to bar_a and bar_b (0 = none).
-        auto issue_s = [&](int i, int st, uint32_t bar_a, uint32_t bar_b) {
-            fav::tc::mma_ss_burst_k128<D / 16>(
-                tmem + C::colS(i), dq0 + (uint64_t)((i * C::kQBytes) >> 4),
-                dk0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_qk, 0u, bar_a, bar_b);
-        };
-        // O_i (+)= P_i V, with P_i read from TMEM (8 columns = 16 keys per k-step) and V MN-major
-        // in shared memory (8-key groups 1024 B apart, 64-column blocks one box apart).
-        auto issue_pv = [&](int i, int st, uint32_t acc, uint32_t bar_a, uint32_t bar_b) {
-            fav::tc::mma_ts_burst_k128(tmem + C::colO(i), tmem + C::colP(i),
-                                       dv0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_pv, acc,
-                                       bar_a, bar_b);
-        };
         // Every lane waits; the outcome is made warp-uniform so that a bounded wait that gives
         // up takes the whole warp out of the loop together (the bursts' elect.sync needs all
         // 32 lanes).
-        auto wait_all = [&](uint32_t bar, uint32_t parity) {
-            return __all_sync(0xffffffffu, fav::mbar_wait(bar, parity, status));
-        };
-        auto try_all = [&](uint32_t bar, uint32_t parity) {
-            return __all_sync(0xffffffffu, fav::mbar_try(bar, parity));
+        // (A non-blocking test first: most of these phases have completed long before.)
+        auto wait_all = [&](uint32_t bar, uint32_t parity) -> bool {
+            if (__all_sync(0xffffffffu, fav::mbar_test(bar, parity))) return true;
+            return __all_sync(0xffffffffu, fav::mbar_wait(bar, parity, status)) != 0;
         };
 #ifdef FAV_TIMING
-        long long ts[16][6];
+        __shared__ long long tsm[32][4];
         const long long t_start = t_ref;
+#define FAV_TSM(g, c) do { if ((g) < 32 && lane == 0) tsm[g][c] = clock64(); } while (0)
+#else
+#define FAV_TSM(g, c) do { } while (0)
 #endif
-        int g = 0;                 // key tiles streamed so far (ring sequence)
-        int np[2] = {0, 0};        // P_i(.) consumed so far, per tile (p_full parity)
-        int nsi[2] = {0, 0};       // S_i(.) issued so far, per tile (s_free parity, kSepP)
-        bool ok = true;
-        for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
-            const Unit U = make_unit(u);
-            const int g0 = g;
-            if constexpr (C::kSepP) {
-                // Weights in their own columns: S_i(j+1) is issued as soon as the softmax has
-                // read S_i(j) (s_free), before P_i(j).V, which is issued when P_i(j) is ready;
-                // the softmax waits for P_i(j).V (p_free) before it stores P_i(j+1) or rescales
-                // O_i.  Each tile's softmax can then run from one key tile to the next without
-                // waiting for the tensor core.
-                const int last0 = U.n_kv_tiles[1] > 0 ? 1 : 0;      // last tile with work
-                if (!(ok = wait_all(k_full + 8 * (g0 % S), (g0 / S) & 1))) break;
-                // S_1(0) waits until tile 0's softmax has reached its exponentials: the two
-                // softmaxes then run half a period apart, so that one's exponentials (MUFU) overlap
-                // the other's loads and maxima instead of competing for the MUFU in lockstep;
-                // the offset carries over to the following key tiles.
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (U.n_kv_tiles[i] == 0) continue;
-                    if (!(ok = wait_all(q_full + 8 * i, k & 1))) break;
-                    if (i == 1 && !(ok = wait_all(s_free, (nsi[0] - 1) & 1))) break;
-                    if (nsi[i] > 0 && !(ok = wait_all(s_free + 8 * i, (nsi[i] - 1) & 1))) break;
-                    fav::tc::fence_after();
-                    issue_s(i, g0 % S, s_full + 8 * i, i == last0 ? k_empty + 8 * (g0 % S) : 0u);
-                    ++nsi[i];
-                }
-                if (!ok) break;
-                if (U.n_kv == 1) fav::tc::commit_elect(q_empty);    // no further S in this unit
-                // Per key tile j, tile by tile: S_i(j+1) (once the softmax has read S_i(j)), then
-                // P_i(j).V_j (once P_i(j) is stored).  Tile 1's softmax runs half a period behind
-                // tile 0's, so this order never holds one tile's MMAs behind the other's events.
-                // K_{j+1} and V_j are released by the last tile's bursts.
-                for (int j = 0; ok && j < U.n_kv; ++j) {
-                    const int gj = g0 + j;
-                    const int st = gj % S, st1 = (gj + 1) % S;
-                    const int last1 = j + 1 < U.n_kv_tiles[1] ? 1 : 0;   // last tile with S(j+1)
-                    const int last = j < U.n_kv_tiles[1] ? 1 : 0;        // last tile with P(j)
-                    bool k_ok = false, v_ok = false;
-#pragma unroll
-                    for (int i = 0; i < 2; ++i) {
-                        if (j + 1 < U.n_kv_tiles[i]) {
-                            if (!k_ok && !(ok = wait_all(k_full + 8 * st1, ((gj + 1) / S) & 1))) break;
-                            k_ok = true;
-                            if (k == 0) FAV_STAMP(ts, j, 3 * i);
-                            if (!(ok = wait_all(s_free + 8 * i, (nsi[i] - 1) & 1))) break;
-                            fav::tc::fence_after();
-                            issue_s(i, st1, s_full + 8 * i, i == last1 ? k_empty + 8 * st1 : 0u);
-                            ++nsi[i];
-                        }
-                        if (j < U.n_kv_tiles[i]) {
-                            if (!v_ok && !(ok = wait_all(v_full + 8 * st, (gj / S) & 1))) break;
-                            v_ok = true;
-                            if (!(ok = wait_all(p_full + 8 * i, np[i] & 1))) break;
-                            ++np[i];
-                            if (k == 0) FAV_STAMP(ts, j, 3 * i + 1);
-                            fav::tc::fence_after();
-                            issue_pv(i, st, j > 0 ? 1u : 0u, p_free + 8 * i, i == last ? v_empty + 8 * st : 0u);
-                            if (j + 1 == U.n_kv_tiles[i]) fav::tc::commit_elect(o_done + 8 * i);
-                            if (k == 0) FAV_STAMP(ts, j, 3 * i + 2);
-                        }
-                    }
-                    if (!ok) break;
-                    // after the unit's last scores (issued in this key tile), its Q buffers can be
-                    // refilled: the commit covers every MMA issued so far
-                    if (j + 2 == U.n_kv) fav::tc::commit_elect(q_empty);
-                }
-                g += U.n_kv;
-                continue;
+        // Scores run two key tiles ahead of the P.V products: (ks, js) is the next tile whose
+        // S is due, Gs its position in the CTA's sequence.
+        int ks = 0, js = 0, Gs = 0;
+        int us = unit_at(0);
+        Unit Us;
+        if (us >= 0) Us = unit(0);
+        // operands of the next S ready (Q of its unit, its K tile)?
+        auto wait_next_s = [&]() -> bool {
+            if (us < 0) return true;
+            if (js == 0 && !wait_all(q_full + 8 * (ks & 1), (ks >> 1) & 1)) return false;
+            return wait_all(k_full + 8 * (Gs % KS), (Gs / KS) & 1);
+        };
+        auto issue_next_s = [&]() {
+            if (us < 0) return;                      // no further tile
+            const int qb = ks & 1, st = Gs % KS;
+            fav::tc::mma_ss_burst_k128<D / 16>(
+                tmem + C::colS(Gs & 1), dq0 + (uint64_t)((qb * C::kQBytes) >> 4),
+                dk0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_qk, 0u, s_full + 8 * (Gs & 1),
+                k_empty + 8 * st);
+            if (js + 1 == Us.n_kv) fav::tc::commit_elect(q_empty + 8 * qb);   // unit's last S
+            ++Gs;
+            if (++js == Us.n_kv) {
+                js = 0;
+                us = unit_at(++ks);
+                if (us >= 0) Us = unit(ks);
             }
-            // first scores of the unit (the previous unit's last P.V are ahead in the pipe, so
-            // S_i(0) cannot overwrite its P_i before it is read)
-            const int last0 = U.n_kv_tiles[1] > 0 ? 1 : 0;      // last tile with work
-            ok = wait_all(q_full, k & 1) && wait_all(k_full + 8 * (g0 % S), (g0 / S) & 1);
-            if (!ok) break;
+        };
+        bool ok = wait_next_s();
+        if (ok) {
             fav::tc::fence_after();
-            issue_s(0, g0 % S, s_full, last0 == 0 ? k_empty + 8 * (g0 % S) : 0u);
-            if (last0 == 1) {
-                if (!(ok = wait_all(q_full + 8, k & 1))) break;
+            issue_next_s();
+            ok = wait_next_s();
+            if (ok) {
                 fav::tc::fence_after();
-                issue_s(1, g0 % S, s_full + 8, k_empty + 8 * (g0 % S));
+                issue_next_s();
             }
-            if (U.n_kv == 1) fav::tc::commit_elect(q_empty);    // no further S in this unit
-            // Issue order per key tile j: [P_0(j).V_j, S_0(j+1)], [P_1(j).V_j, S_1(j+1)]: the
-            // scores of the two tiles arrive half a period apart, so each softmax runs while the
-            // tensor core works on the other tile.  The stage releases (v_empty, k_empty) are
-            // committed by the bursts of the last tile with work in this key tile.
-            for (int j = 0; ok && j < U.n_kv; ++j) {
-                const int gj = g0 + j;
-                const int st = gj % S, st1 = (gj + 1) % S;
-                const bool nxt = j + 1 < U.n_kv;
-                const int last = j < U.n_kv_tiles[1] ? 1 : 0;
-                // tested ahead: V_j now, K_{j+1} before the first burst
-                bool v_ready = try_all(v_full + 8 * st, (gj / S) & 1);
-                bool k_ready = !nxt;
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (j >= U.n_kv_tiles[i]) continue;
-                    if (k == 0) FAV_STAMP(ts, j, 3 * i);
-                    if (!wait_all(p_full + 8 * i, np[i] & 1)) { ok = false; break; }
-                    ++np[i];
-                    if (!v_ready) {
-                        if (!wait_all(v_full + 8 * st, (gj / S) & 1)) { ok = false; break; }
-                        v_ready = true;
-                    }
-                    if (k == 0) FAV_STAMP(ts, j, 3 * i + 1);
-                    fav::tc::fence_after();
-                    const bool k_tested = k_ready || try_all(k_full + 8 * st1, ((gj + 1) / S) & 1);
-                    const bool more = j + 1 < U.n_kv_tiles[i];          // S_i(j+1) follows
-                    issue_pv(i, st, j > 0 ? 1u : 0u, i == last ? v_empty + 8 * st : 0u,
-                             more ? 0u : o_done + 8 * i);
-                    if (more) {
-                        if (!k_tested && !wait_all(k_full + 8 * st1, ((gj + 1) / S) & 1)) {
-                            ok = false;
-                            break;
-                        }
-                        k_ready = true;
-                        fav::tc::fence_after();
-                        issue_s(i, st1, s_full + 8 * i, i == last ? k_empty + 8 * st1 : 0u);
-                    } else if (i == last && nxt) {
-                        fav::tc::commit_elect(k_empty + 8 * st1);   // another tile read K_{j+1}
-                    }
-                    if (k == 0) FAV_STAMP(ts, j, 3 * i + 2);
-                }
-                // after the unit's last scores (issued in this key tile), its Q buffers can be
-                // refilled: the commit covers every MMA issued so far
-                if (ok && j + 2 == U.n_kv) fav::tc::commit_elect(q_empty);
-            }
-            g += U.n_kv;
-#ifdef FAV_TIMING
-            if (k == 0 && blockIdx.x == 0 && lane == 0)
-                for (int j = 0; j < min(U.n_kv, 16); ++j)
-                    printf("[mma] j=%2d wait_p0 %6lld got_p0 %6lld done0 %6lld | wait_p1 %6lld got_p1 %6lld done1 %6lld\n", j,
-                           ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start, ts[j][3] - t_start,
-                           ts[j][4] - t_start, ts[j][5] - t_start);
-#endif
         }
+        // The issuing lane blocks until the tensor pipe has taken most of a burst, so a wait
+        // placed right after a burst overlaps the MMAs still queued, while one placed before a
+        // burst that the pipe is waiting for leaves it idle.  Per key tile G: the weights,
+        // P(G).V, then (behind it) K(G+2) / Q and V(G+1), then S(G+2).
+        int Gp = 0;
+        if (ok) ok = wait_all(v_full, 0);            // V(0)
+        for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
+            const Unit U = unit(k);
+            const bool more_units = unit_at(k + 1) >= 0;
+            for (int j = 0; j < U.n_kv; ++j, ++Gp) {
+                const int vs = Gp % VS;
+                FAV_TSM(Gp, 0);
+                if (!(ok = wait_all(p_full + 8 * (Gp & 1), (Gp >> 1) & 1))) break;
+                FAV_TSM(Gp, 1);
+                fav::tc::fence_after();
+                fav::tc::mma_pv_split<NS>(tmem + C::kColO, tmem + C::colS(Gp & 1),
+                                          dv0 + (uint64_t)((vs * C::kKVBytes) >> 4), idesc_pv,
+                                          j > 0 ? 1u : 0u, v_empty + 8 * vs, pv_done);
+                if (j + 1 == U.n_kv) fav::tc::commit_elect(o_done);   // the unit's O is final
+                FAV_TSM(Gp, 2);
+                if (!(ok = wait_next_s())) break;
+                if (j + 1 < U.n_kv || more_units) {
+                    const int g1 = Gp + 1;
+                    if (!(ok = wait_all(v_full + 8 * (g1 % VS), (g1 / VS) & 1))) break;
+                }
+                fav::tc::fence_after();
+                issue_next_s();
+                FAV_TSM(Gp, 3);
+            }
+        }
+#ifdef FAV_TIMING
+        if (blockIdx.x == 0 && lane == 0)
+            for (int g = 0; g < min(Gp, 32); ++g)
+                printf("[mma] G=%2d start %6lld got_p %6lld pv_issued %6lld s_issued %6lld\n", g,
+                       tsm[g][0] - t_start, tsm[g][1] - t_start, tsm[g][2] - t_start, tsm[g][3] - t_start);
+#endif
+#undef FAV_TSM
     } else {
-        // ---------------- softmax / correction / epilogue: one thread per query row ----------------
-        const int i = warp >> 2;                          // query tile of this warpgroup
-        const int quarter = warp & 3;
+        // ---------------- softmax / correction / epilogue: one thread per query row and split ----------------
+        const int quarter = warp & 3, split = warp >> 2;
         const int row = quarter * 32 + lane;
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
-        const uint32_t colS = i ? C::colS(1) : C::colS(0);
-        const uint32_t colO = i ? C::colO(1) : C::colO(0);
-        int ns = 0, no = 0;        // S_i(.) and O_i completions consumed so far (parities)
-        int npst = 0;              // P_i(.) stored so far (kSepP: p_free parity)
-        const uint32_t colP = i ? C::colP(1) : C::colP(0);
+        const uint32_t colO = C::kColO + split * D;
+        int Gt = 0;                // key tiles consumed so far (the CTA's sequence)
         bool ok = true;
 #ifdef FAV_TIMING
-        long long ts[16][6];
+        long long ts[32][5];
+        long long te[8], te1[8], te2[8], te3[8];
         const long long t_start = t_ref;
+#define FAV_TSS(c) do { if (Gt < 32) ts[Gt][c] = clock64(); } while (0)
+#else
+#define FAV_TSS(c) do { } while (0)
 #endif
+        // Epilogue of unit kk (running maximum m, sum l of this row and split): merge the
+        // splits, O / L, LSE.  It runs after the next unit's first weights are stored (so that
+        // the wait for the unit's last P.V overlaps that softmax) and before they are released
+        // (the next unit's first P.V overwrites every O_s).
+        auto epilogue = [&](const Unit &U, float m, float l, int kk) -> bool {
+            if (!__all_sync(~0u, fav::mbar_wait(o_done, kk & 1, status))) return false;
+#ifdef FAV_TIMING
+            if (kk < 8) te1[kk] = clock64();
+#endif
+            fav::tc::fence_after();
+            // (m_s, l_s) of this row's splits through shared memory (slot kk % 2)
+            const int xs = kk & 1;
+            float2 *xrow = xch + ((xs * 4 + quarter) * NS) * 32 + lane;
+            xrow[split * 32] = make_float2(m, l);
+            fav::mbar_arrive(xch_bar + 8 * (xs * 4 + quarter));
+            if (!__all_sync(~0u, fav::mbar_wait(xch_bar + 8 * (xs * 4 + quarter), (kk >> 1) & 1, status)))
+                return false;
+#ifdef FAV_TIMING
+            if (kk < 8) te2[kk] = clock64();
+#endif
+            float Mx = -INFINITY;
+            float2 ml[NS];
+#pragma unroll
+            for (int t = 0; t < NS; ++t) {
+                ml[t] = xrow[t * 32];
+                Mx = fmaxf(Mx, ml[t].x);
+            }
+            float w[NS], L = 0.f;
+#pragma unroll
+            for (int t = 0; t < NS; ++t) {
+                w[t] = (ml[t].x == -INFINITY) ? 0.f : fav::fast_exp2(ml[t].x - Mx);
+                L += w[t] * ml[t].y;
+            }
+            const int qi = U.t * BM + row;
+            const float vsc = kV16 ? v_scale[U.b * Hkv + U.kvh] : 1.f;   // V = v_scale * (fp16 copy)
+            const float inv_l = vsc / L;
+            // This warp's columns [split * 64, split * 64 + 64) of O -- one 64-column block of
+            // the tile -- go to the unit's Q buffer (free: the unit's S products have completed)
+            // in the TMA box layout (rows of 128 bytes, 16-byte chunks XOR-swizzled by row % 8);
+            // the store warp writes the tile out with one TMA store (rows beyond Nq are not
+            // written).
+            const uint32_t stage = sQ + (kk & 1) * C::kQBytes + split * (BM * 128) + row * 128;
+#ifdef FAV_TIMING
+            if (kk < 8) te3[kk] = clock64();
+#endif
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                static_assert(NS == 2, "two accumulators per chunk");
+                uint32_t v0[32], v1[32];
+                fav::tc::ld_32x32b_x32(trow + C::kColO + split * 64 + c * 32, v0);
+                fav::tc::ld_32x32b_x32(trow + C::kColO + D + split * 64 + c * 32, v1);
+                fav::tc::wait_ld_dep(v0);
+                fav::tc::wait_ld_dep(v1);
+                float acc[32];
+#pragma unroll
+                for (int e = 0; e < 32; ++e)
+                    acc[e] = fmaf(w[0], __uint_as_float(v0[e]), w[1] * __uint_as_float(v1[e]));
+#pragma unroll
+                for (int e = 0; e < 32; e += 8) {
+                    const uint32_t x0 = fav::Elem<T>::pack(acc[e] * inv_l, acc[e + 1] * inv_l);
+                    const uint32_t x1 = fav::Elem<T>::pack(acc[e + 2] * inv_l, acc[e + 3] * inv_l);
+                    const uint32_t x2 = fav::Elem<T>::pack(acc[e + 4] * inv_l, acc[e + 5] * inv_l);
+                    const uint32_t x3 = fav::Elem<T>::pack(acc[e + 6] * inv_l, acc[e + 7] * inv_l);
+                    const uint32_t chunk = (uint32_t)(c * 4 + e / 8) ^ (uint32_t)(row & 7);
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};"
+                                 ::"r"(stage + (chunk << 4)), "r"(x0), "r"(x1), "r"(x2), "r"(x3)
+                                 : "memory");
+                }
+            }
+            fav::tc::fence_proxy_async_smem();   // visible to the TMA store (async proxy)
+            fav::mbar_arrive(o_staged + 8 * (kk & 1));
+            if (split == 0 && qi < Nq && lse)
+                lse[(long long)(U.b * Hq + U.h) * Nq + qi] = (Mx - kPShift + log2f(L)) * kLn2;
+#ifdef FAV_TIMING
+            if (kk < 8) te[kk] = clock64();
+#endif
+            return true;
+        };
+        int k_pend = -1;           // unit whose epilogue is still due
+        Unit U_pend;
+        float m_pend = 0.f, l_pend = 0.f;
         for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
-            const Unit U = make_unit(u);
-            const int n_mine = U.n_kv_tiles[i];
-            if (n_mine == 0) continue;
-            const int ti = U.t[i], hi = U.h[i];
-            const int q0 = ti * BM;
+            const Unit U = unit(k);
+            const int q0 = U.t * BM;
             const int qi = q0 + row;                          // query index of this row
             const int lim = causal ? min(Nkv, qi + off + 1) : Nkv;       // visible keys: [0, lim)
             const int lim_tile = causal ? min(Nkv, q0 + off + 1) : Nkv;  // smallest lim in the tile
             float m = -INFINITY, l = 0.f;
-            for (int j = 0; j < n_mine; ++j) {
-                if (k == 0) FAV_STAMP(ts, j, 0);
-                if (!__all_sync(~0u, fav::mbar_wait(s_full + 8 * i, ns & 1, status))) { ok = false; break; }
-                ++ns;
-                if (k == 0) FAV_STAMP(ts, j, 1);
+            for (int j = 0; j < U.n_kv; ++j, ++Gt) {
+                FAV_TSS(0);
+                if (!__all_sync(~0u, fav::mbar_wait(s_full + 8 * (Gt & 1), (Gt >> 1) & 1, status))) {
+                    ok = false;
+                    break;
+                }
+                FAV_TSS(1);
                 fav::tc::fence_after();
-                const int key0 = j * BN;
-                const bool crosses = key0 + BN > lim_tile;   // tile crosses the diagonal or the end
-                float s[BN];
-                // S row from TMEM (and the mask: keys at or beyond lim get -inf)
-                auto load_s = [&]() {
-                    uint32_t r[BN / 32][32];
+                const uint32_t colS = C::colS(Gt & 1) + split * SK;
+                const int key0 = j * BN + split * SK;
+                const bool crosses = key0 + SK > lim_tile;   // the split crosses the diagonal or the end
+                float s[SK];
+                // scores of this split from TMEM (and the mask: keys at or beyond lim get -inf)
+                {
+                    uint32_t r[SK / 32][32];
 #pragma unroll
-                    for (int c = 0; c < BN / 32; ++c) fav::tc::ld_32x32b_x32(trow + colS + c * 32, r[c]);
+                    for (int c = 0; c < SK / 32; ++c) fav::tc::ld_32x32b_x32(trow + colS + c * 32, r[c]);
 #pragma unroll
-                    for (int c = 0; c < BN / 32; ++c) fav::tc::wait_ld_dep(r[c]);
+                    for (int c = 0; c < SK / 32; ++c) fav::tc::wait_ld_dep(r[c]);
 #pragma unroll
-                    for (int c = 0; c < BN; ++c) s[c] = __uint_as_float(r[c >> 5][c & 31]);
+                    for (int c = 0; c < SK; ++c) s[c] = __uint_as_float(r[c >> 5][c & 31]);
                     if (crosses) {
+                        const int nvis = lim - key0;              // keys [0, nvis) of the split visible
 #pragma unroll
-                        for (int c = 0; c < BN; ++c)
-                            if (key0 + c >= lim) s[c] = -INFINITY;
+                        for (int c = 0; c < SK; ++c)
+                            if (c >= nvis) s[c] = -INFINITY;
                     }
-                };
-                // raw row maximum: 8 independent chains of 3-input max, then a tree
-                auto row_max = [&]() {
+                }
+                // raw maximum of the split: 8 independent chains of 3-input max, then a tree
+                float mx;
+                {
                     float m8[8];
 #pragma unroll
                     for (int c = 0; c < 8; ++c) m8[c] = s[c];
 #pragma unroll
-                    for (int c = 8; c < BN; c += 16) {
+                    for (int c = 8; c < SK; c += 16) {
 #pragma unroll
-                        for (int q = 0; q < 8; ++q) m8[q] = fav::fmax3(m8[q], s[c + q], s[c + 8 + q]);
+                        for (int q = 0; q < 8; ++q)
+                            m8[q] = (c + 8 < SK) ? fav::fmax3(m8[q], s[c + q], s[c + 8 + q])
+                                                 : fmaxf(m8[q], s[c + q]);
                     }
-                    return fav::fmax3(fav::fmax3(m8[0], m8[1], m8[2]), fav::fmax3(m8[3], m8[4], m8[5]),
-                                      fmaxf(m8[6], m8[7]));
-                };
-                // p = exp2(s * scale_log2 - mref) on pairs (one packed FMA, two ex2, one packed
-                // add), fp16 weights stored to TMEM half a row at a time (keys [64h, 64h + 64)
-                // over S columns [32h, 32h + 32), whose scores are already in registers); the
-                // fp32 sum goes to psum.
-                float psum = 0.f;
-                auto exp_store = [&](float mref) {
+                    mx = fav::fmax3(fav::fmax3(m8[0], m8[1], m8[2]), fav::fmax3(m8[3], m8[4], m8[5]),
+                                    fmaxf(m8[6], m8[7])) * scale_log2;
+                }
+                FAV_TSS(2);
+                // lazy rescale: move the reference maximum only when it grows by > 2^4
+                float alpha = 1.f;
+                bool rescale = false;
+                if (mx > m + kRescaleThreshold) {
+                    alpha = fav::fast_exp2(m - mx);   // 0 while m = -inf
+                    rescale = (j > 0);
+                    m = mx;
+                    l *= alpha;
+                }
+                // weights p = exp2(s * scale_log2 - mref) on pairs (one packed FMA, two ex2, one
+                // packed add), stored as fp16 over the split's first SK / 2 score columns (read
+                // above); a split with no visible key so far (m = -inf) stores zeros.
+                {
+                    const float mref = (m == -INFINITY) ? 0.f : m - kPShift;
                     const float2 sc2 = make_float2(scale_log2, scale_log2);
                     const float2 nm2 = make_float2(-mref, -mref);
                     float2 l4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-                    static_for<0, 2>([&](auto hc) {
-                        constexpr int h = decltype(hc)::value;
-                        uint32_t pk[32];
-                        static_for<0, 32>([&](auto pc) {
-                            constexpr int e = 2 * decltype(pc)::value;
-                            constexpr int c = 64 * h + e;
-                            const float2 x = fav::ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
-                            const float2 p = exp2_pair<c / 2>(x);
-                            l4[(e >> 1) & 3] = fav::fadd2(l4[(e >> 1) & 3], p);
-                            pk[e >> 1] = fav::Elem<TP>::pack(p.x, p.y);
-                        });
-                        fav::tc::st_32x32b_x32(trow + colP + 32 * h, pk);
+                    uint32_t pk[SK / 2];
+                    static_for<0, SK / 2>([&](auto pc) {
+                        constexpr int e = decltype(pc)::value;
+                        const float2 x = fav::ffma2(make_float2(s[2 * e], s[2 * e + 1]), sc2, nm2);
+                        const float2 p = make_float2(fav::fast_exp2(x.x), fav::fast_exp2(x.y));
+                        l4[e & 3] = fav::fadd2(l4[e & 3], p);
+                        pk[e] = fav::Elem<TP>::pack(p.x, p.y);
                     });
+                    fav::tc::st_32x32b_x32(trow + colS, pk);
                     const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
-                    psum = a.x + a.y;
-                };
-                float alpha = 1.f;
-                bool rescale = false;
-                // lazy rescale: move the reference maximum only when it grows by > 2^4
-                auto move_max = [&](float mx) {
-                    if (mx > m + kRescaleThreshold) {
-                        alpha = fav::fast_exp2(m - mx);   // 0 on the first tile (m = -inf)
-                        rescale = (j > 0);
-                        m = mx;
-                        l *= alpha;
-                    }
-                };
-                // two passes: the row maximum, then the weights against the (lazy) reference
-                load_s();
-                if (k == 0) FAV_STAMP(ts, j, 2);
-                move_max(row_max() * scale_log2);
-                if (k == 0) FAV_STAMP(ts, j, 3);
-                if constexpr (C::kSepP) {
-                    // S_i has been read (long ago; the signal waits for the start of the
-                    // exponentials, which also paces the other tile: see the MMA warp)
-                    fav::tc::fence_before();
-                    __syncwarp();
-                    if (lane == 0) fav::mbar_arrive(s_free + 8 * i);
+                    l += a.x + a.y;
                 }
-                // P_i over the first 64 columns of S_i (two 16-bit weights per column)
-                if constexpr (C::kSepP) {
-                    // P_i's columns and O_i are free and stable once the previous P_i.V is done
-                    if (npst > 0 && !__all_sync(~0u, fav::mbar_wait(p_free + 8 * i, (npst - 1) & 1, status))) {
+                FAV_TSS(3);
+                // O_s *= alpha, once P(G-1).V (the last product into O_s) has completed.  S(G)
+                // was issued after P(G-2).V and has completed, so pv_done has completed phase
+                // G-2 and cannot have completed G (that needs these weights): the parity of phase
+                // G-1 is unambiguous.
+                if (__any_sync(~0u, rescale)) {
+                    if (!__all_sync(~0u, fav::mbar_wait(pv_done, (Gt - 1) & 1, status))) {
                         ok = false;
                         break;
                     }
                     fav::tc::fence_after();
-                }
-                ++npst;
-                exp_store(m - kPShift);
-                l += psum;
-                if (k == 0) FAV_STAMP(ts, j, 4);
-                // O_i is stable here: P_i(j-1).V has completed (D = 128: it was issued before
-                // S_i(j) and MMAs complete in issue order; D = 64: the p_free wait above).
-                if (__any_sync(~0u, rescale)) {
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
                         const uint32_t col = colO + c * 32;
@@ -605,140 +614,46 @@ fav_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                         fav::tc::st_32x32b_x32(trow + col, v);
                     }
                 }
+                // the previous unit's epilogue, between this unit's first weights and their release
+                if (j == 0 && k_pend >= 0) {
+                    if (!epilogue(U_pend, m_pend, l_pend, k_pend)) {
+                        ok = false;
+                        break;
+                    }
+                    k_pend = -1;
+                }
                 fav::tc::wait_st();
                 fav::tc::fence_before();
                 __syncwarp();
-                if (lane == 0) fav::mbar_arrive(p_full + 8 * i);
-                if (k == 0) FAV_STAMP(ts, j, 5);
+                if (lane == 0) fav::mbar_arrive(p_full + 8 * (Gt & 1));
+                FAV_TSS(4);
             }
-#ifdef FAV_TIMING
-            if (k == 0 && blockIdx.x == 0 && (threadIdx.x & 127) == 0)
-                for (int j = 0; j < min(n_mine, 16); ++j)
-                    printf("[sm%d] j=%2d wait %6lld s_ready %6lld ld %6lld max %6lld exp %6lld arrive %6lld\n",
-                           i, j, ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start,
-                           ts[j][3] - t_start, ts[j][4] - t_start, ts[j][5] - t_start);
-#endif
             if (!ok) break;
-            // ---------------- epilogue: O / l, LSE ----------------
-            // (the next unit's first P.V, which overwrites O_i, waits for this warpgroup's next
-            // P_i: it cannot run before these loads)
-            if (!__all_sync(~0u, fav::mbar_wait(o_done + 8 * i, no & 1, status))) { ok = false; break; }
-            ++no;
-            fav::tc::fence_after();
-            const float vsc = kV16 ? v_scale[U.bkv] : 1.f;     // V = v_scale * (fp16 copy)
-            const float inv_l = vsc / l;
-            const bool valid = qi < Nq;
-            T *orow = o + U.b * os.b + hi * os.h + (long long)qi * os.n;
-#pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t v[32];
-                fav::tc::ld_32x32b_x32(trow + colO + c * 32, v);
-                fav::tc::wait_ld_dep(v);
-                if (valid) {
-#pragma unroll
-                    for (int e = 0; e < 32; e += 8) {
-                        uint4 v4;
-                        v4.x = fav::Elem<T>::pack(__uint_as_float(v[e]) * inv_l, __uint_as_float(v[e + 1]) * inv_l);
-                        v4.y = fav::Elem<T>::pack(__uint_as_float(v[e + 2]) * inv_l, __uint_as_float(v[e + 3]) * inv_l);
-                        v4.z = fav::Elem<T>::pack(__uint_as_float(v[e + 4]) * inv_l, __uint_as_float(v[e + 5]) * inv_l);
-                        v4.w = fav::Elem<T>::pack(__uint_as_float(v[e + 6]) * inv_l, __uint_as_float(v[e + 7]) * inv_l);
-                        *reinterpret_cast<uint4 *>(orow + c * 32 + e) = v4;
-                    }
-                }
-            }
-            if (valid && lse) lse[(long long)(U.b * Hq + hi) * Nq + qi] = (m - kPShift + log2f(l)) * kLn2;
-            fav::tc::fence_before();
+            k_pend = k;
+            U_pend = U;
+            m_pend = m;
+            l_pend = l;
         }
+        if (ok && k_pend >= 0) (void)epilogue(U_pend, m_pend, l_pend, k_pend);
+#ifdef FAV_TIMING
+        if (blockIdx.x == 0 && (threadIdx.x & 127) == 0) {
+            for (int g = 0; g < min(Gt, 32); ++g)
+                printf("[sm%d] G=%2d wait %6lld s_ready %6lld max %6lld exp %6lld arrive %6lld\n",
+                       split, g, ts[g][0] - t_start, ts[g][1] - t_start, ts[g][2] - t_start,
+                       ts[g][3] - t_start, ts[g][4] - t_start);
+            for (int kk = 0; kk < 3; ++kk)
+                printf("[epi%d] unit %d o_done %6lld xch %6lld merged %6lld done %6lld\n", split, kk,
+                       te1[kk] - t_start, te2[kk] - t_start, te3[kk] - t_start, te[kk] - t_start);
+        }
+#endif
+#undef FAV_TSS
     }
 
     fav::tc::fence_before();
     __syncthreads();
     fav::tc::fence_after();
-    if (warp == kMmaWarp) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
+    if (warp == C::kMmaWarp) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
 }
-
-// ---- bf16 V -> fp16 V (per-KV-head power-of-two scale), for the kV16 kernel ----
-// Pass 1: per KV head, the largest finite |v| (as float bits: non-negative floats order like
-// their bit patterns, so an unsigned atomicMax finds it).
-// V rows are read through its strides (element offsets of head (b, g): b * vs.b + g * vs.h,
-// row n: + n * vs.n), D / 8 16-byte chunks per row.
-__device__ __forceinline__ const uint4 *fav_v_chunk(const uint16_t *v, FavStrides vs, int Hkv,
-                                                    long long head, long long i, int d8) {
-    const long long b = head / Hkv, g = head % Hkv, n = i / d8, c = i % d8;
-    return reinterpret_cast<const uint4 *>(v + b * vs.b + g * vs.h + n * vs.n + c * 8);
-}
-
-__global__ void __launch_bounds__(256)
-fav_vmax_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
-                unsigned *__restrict__ vmax_bits, long long per_head) {
-    const long long head = blockIdx.y;
-    unsigned mx = 0;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_head;
-         i += (long long)gridDim.x * blockDim.x) {
-        const uint4 w = *fav_v_chunk(v, vs, Hkv, head, i, d8);
-        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            // two bf16 values: |x| bits are the low 15 bits of each half, moved to float bits
-            const uint32_t lo = (u[k] & 0x7FFFu) << 16, hi = u[k] & 0x7FFF0000u;
-            if (lo < 0x7F800000u) mx = max(mx, lo);      // finite only
-            if (hi < 0x7F800000u) mx = max(mx, hi);
-        }
-    }
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) mx = max(mx, __shfl_xor_sync(~0u, mx, d));
-    if ((threadIdx.x & 31) == 0 && mx) atomicMax(vmax_bits + head, mx);
-}
-
-// Scale exponent of a head: e = floor(log2(max|v|)) - 14, so that max|v| * 2^-e < 2^15 (fp16
-// max 65504); a head of zeros keeps e = 0.  Clamped to [-126, 127] so that 2^e and 2^-e are
-// both finite normal floats (a head whose maximum is below 2^-112 is scaled by 2^126 only).
-__device__ __forceinline__ int fav_v16_exponent(unsigned vmax_bits) {
-    if (vmax_bits == 0) return 0;
-    const int e2 = (int)(vmax_bits >> 23) - 127;        // floor(log2), -127 for subnormals
-    return min(127, max(-126, e2 - 14));
-}
-
-// Pass 2: v16 = fp16(v * 2^-e).  A bf16 value has 8 significant bits, which fp16 holds exactly
-// down to 2^-17 (subnormals included), so every |v| >= 2^(e-17) -- everything within about
-// 2^-31 of the head's maximum -- converts exactly; smaller values err by less than 2^(e-25).
-// Non-finite values stay non-finite.  Also stores v_scale = 2^e.
-__global__ void __launch_bounds__(256)
-fav_v16_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
-               uint4 *__restrict__ v16, const unsigned *__restrict__ vmax_bits,
-               float *__restrict__ v_scale, long long per_head) {
-    const long long head = blockIdx.y;
-    const int e = fav_v16_exponent(vmax_bits[head]);
-    if (blockIdx.x == 0 && threadIdx.x == 0) v_scale[head] = ldexpf(1.f, e);
-    const float inv = ldexpf(1.f, -e);
-    uint4 *dst = v16 + head * per_head;        // contiguous [B, Hkv, Nkv, D]
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_head;
-         i += (long long)gridDim.x * blockDim.x) {
-        const uint4 w = *fav_v_chunk(v, vs, Hkv, head, i, d8);
-        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
-        uint32_t r[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const float lo = __uint_as_float(u[k] << 16) * inv;
-            const float hi = __uint_as_float(u[k] & 0xFFFF0000u) * inv;
-            r[k] = fav::Elem<__half>::pack(lo, hi);
-        }
-        dst[i] = make_uint4(r[0], r[1], r[2], r[3]);
-    }
-}
-
-// workspace of the kV16 path: [fp16 V][vmax bits per KV head][scale per KV head]
-struct V16Layout {
-    size_t v16, vmax, scale, total;
-    explicit V16Layout(const FavArgs &a) {
-        const size_t heads = (size_t)a.B * a.Hkv;
-        auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
-        v16 = 0;
-        vmax = up(heads * a.Nkv * a.D * 2);
-        scale = vmax + up(heads * 4);
-        total = scale + up(heads * 4);
-    }
-};
 
 template <typename T, int D, bool kV16>
 fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
@@ -747,55 +662,41 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
     FavStrides vstr = a.vs;
     const float *v_scale = nullptr;
     if constexpr (kV16) {
-        if (!workspace) return FAV_ERR_NO_MEMORY;
-        const V16Layout L(a);
-        uint8_t *ws = static_cast<uint8_t *>(workspace);
-        unsigned *vmax = reinterpret_cast<unsigned *>(ws + L.vmax);
-        float *vsc = reinterpret_cast<float *>(ws + L.scale);
-        const long long heads = (long long)a.B * a.Hkv;
-        const long long per_head = (long long)a.Nkv * a.D / 8;      // uint4 chunks (D % 8 == 0)
-        if (heads > 65535) return FAV_ERR_UNSUPPORTED;
-        const unsigned bx = (unsigned)std::max<long long>(
-            1, std::min<long long>((per_head + 255) / 256, std::max<long long>(1, 4LL * a.num_sms / heads)));
-        if (cudaMemsetAsync(vmax, 0, heads * sizeof(unsigned), stream) != cudaSuccess)
-            return FAV_ERR_CUDA;
-        fav_vmax_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(
-            static_cast<const uint16_t *>(a.v), a.vs, a.Hkv, D / 8, vmax, per_head);
-        fav_v16_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(
-            static_cast<const uint16_t *>(a.v), a.vs, a.Hkv, D / 8,
-            reinterpret_cast<uint4 *>(ws + L.v16), vmax, vsc, per_head);
-        if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_v16_kernel", stream))
-            return FAV_ERR_CUDA;
-        vsrc = ws + L.v16;
-        vstr = fav_contiguous_strides(a.Hkv, a.Nkv, D);
-        v_scale = vsc;
+        const fav_status st = fav_v16_convert(a, workspace, stream, &vsrc, &vstr, &v_scale);
+        if (st != FAV_OK) return st;
     }
-    alignas(64) CUtensorMap tmQ, tmK, tmV;
-    fav_status st = fav_make_tmap_4d(&tmQ, a.q, D, a.Nq, a.Hq, a.B, a.qs, BM);
-    if (st == FAV_OK) st = fav_make_tmap_4d(&tmK, a.k, D, a.Nkv, a.Hkv, a.B, a.ks, BN);
-    if (st == FAV_OK) st = fav_make_tmap_4d(&tmV, vsrc, D, a.Nkv, a.Hkv, a.B, vstr, BN);
+    alignas(64) CUtensorMap tmQ, tmK, tmV, tmO;
+    fav_status st = fav_make_tmap_tiles(&tmQ, a.q, D, a.Nq, a.Hq, a.B, a.qs, BM);
+    if (st == FAV_OK) st = fav_make_tmap_tiles(&tmK, a.k, D, a.Nkv, a.Hkv, a.B, a.ks, BN);
+    if (st == FAV_OK) st = fav_make_tmap_tiles(&tmV, vsrc, D, a.Nkv, a.Hkv, a.B, vstr, BN);
+    if (st == FAV_OK) st = fav_make_tmap_tiles(&tmO, a.o, D, a.Nq, a.Hq, a.B, a.os, BM);
     if (st != FAV_OK) return st;
-    auto kern = fav_prefill_kernel<T, D, kV16>;
+    auto kern = fav_prefill_split_kernel<T, D, kV16>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
         cudaSuccess)
         return FAV_ERR_CUDA;
     const int n_qtiles = (a.Nq + BM - 1) / BM;
-    const int G = a.Hq / a.Hkv;
-    const int pair_heads = (G % 2 == 0) ? 1 : 0;
-    const long long units = pair_heads ? (long long)n_qtiles * a.B * (a.Hq / 2)
-                                       : (long long)((n_qtiles + 1) / 2) * a.B * a.Hq;
-    if (units > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
+    const long long units = (long long)n_qtiles * a.B * a.Hq;
+    // (unit indices up to units + grid size are formed in int)
+    if (units + a.num_sms > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
     // persistent: one CTA per SM at most, each working through its share of the units
-    const long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
-    kern<<<(unsigned)blocks, kThreads, C::kSmemBytes, stream>>>(
-        tmQ, tmK, tmV, (T *)a.o, a.os, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
-        pair_heads, a.scale * kLog2e, a.causal, a.dev_status);
-    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_kernel", stream))
+    long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
+    if (a.prefill_grid > 0) blocks = std::min<long long>(blocks, a.prefill_grid);
+    kern<<<(unsigned)blocks, C::kThreads, C::kSmemBytes, stream>>>(
+        tmQ, tmK, tmV, tmO, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
+        a.scale * kLog2e, a.causal, a.dev_status);
+    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_split_kernel", stream))
         return FAV_ERR_CUDA;
     return FAV_OK;
 }
 
 }  // namespace
+
+fav_status fav_launch_prefill_split(const FavArgs &a, void *workspace, cudaStream_t s) {
+    if (a.D != 128) return FAV_ERR_UNSUPPORTED;
+    return a.dtype == FAV_F16 ? launch<__half, 128, false>(a, workspace, s)
+                              : launch<__nv_bfloat16, 128, true>(a, workspace, s);
+}
 
 bool fav_prefill_supported(const FavArgs &a) {
     if (a.dtype != FAV_F16 && a.dtype != FAV_BF16) return false;
@@ -804,13 +705,12 @@ bool fav_prefill_supported(const FavArgs &a) {
 }
 
 size_t fav_prefill_workspace_bytes(const FavArgs &a) {
-    return a.dtype == FAV_BF16 ? V16Layout(a).total : 0;
+    return a.dtype == FAV_BF16 ? fav_v16_workspace_bytes(a) : 0;
 }
 
+// D = 128: the key-split kernel above; D = 64: the two-tile kernel (fav_prefill_pair.cu).  Each
+// design is the faster one at its head dimension (measured on the prefill workloads).
 fav_status fav_launch_prefill(const FavArgs &a, void *workspace, cudaStream_t s) {
-    if (a.dtype == FAV_F16)
-        return a.D == 128 ? launch<__half, 128, false>(a, workspace, s)
-                          : launch<__half, 64, false>(a, workspace, s);
-    return a.D == 128 ? launch<__nv_bfloat16, 128, true>(a, workspace, s)
-                      : launch<__nv_bfloat16, 64, true>(a, workspace, s);
+    return a.D == 128 ? fav_launch_prefill_split(a, workspace, s)
+                      : fav_launch_prefill_pair(a, workspace, s);
 }

@@ -157,6 +157,39 @@ __device__ __forceinline__ void mma_ts_burst_k128(uint32_t d_tmem, uint32_t a_tm
         : "memory");
 }
 #undef FAV_MMA_TS_STEP
+
+// One step of a split P.V burst: D at %0 + DOFF columns, A (weights) at %1 + AOFF columns, B
+// at descriptor %2 + BOFF (16-byte units), accumulate predicate PRED.
+#define FAV_MMA_PV_STEP(DOFF, AOFF, BOFF, PRED)                                  \
+    "add.u32 td, %0, " #DOFF ";\n\tadd.u32 ta, %1, " #AOFF ";\n\t"           \
+    "add.s64 b1, %2, " #BOFF ";\n\t"                                          \
+    "@e tcgen05.mma.cta_group::1.kind::f16 [td], [ta], b1, %3, " #PRED ";\n\t"
+
+// O_s (+)= P_s V_s for the NSPLIT (= 2) key splits of a 128-key tile, in one burst: split s has its
+// own accumulator of D columns at d_tmem + s * D, its weights (128 / NSPLIT keys, two per
+// column) at a_tmem + s * (128 / NSPLIT) and its V rows (MN-major, 128 bytes per key row) at
+// s * (128 / NSPLIT) * 128 bytes past bdesc.  k-steps of 16 keys: A +8 columns, B +2048 bytes.
+// `acc` = 0 overwrites each accumulator with its first MMA.
+template <int NSPLIT>
+__device__ __forceinline__ void mma_pv_split(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                             uint32_t idesc, uint32_t acc, uint32_t bar_a = 0,
+                                             uint32_t bar_b = 0) {
+    static_assert(NSPLIT == 2, "key splits (D = 128)");
+    if constexpr (NSPLIT == 2) {   // D = 128: 64 keys per split, 4 k-steps
+        asm volatile(
+            "{\n\t.reg .pred e, p, t, ca, cb;\n\t.reg .b32 td, ta;\n\t.reg .b64 b1;\n\t"
+            "elect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\tsetp.eq.b32 t, %4, %4;\n\t"
+            FAV_MMA_PV_STEP(0, 0, 0, p) FAV_MMA_PV_STEP(0, 8, 128, t)
+            FAV_MMA_PV_STEP(0, 16, 256, t) FAV_MMA_PV_STEP(0, 24, 384, t)
+            FAV_MMA_PV_STEP(128, 64, 512, p) FAV_MMA_PV_STEP(128, 72, 640, t)
+            FAV_MMA_PV_STEP(128, 80, 768, t) FAV_MMA_PV_STEP(128, 88, 896, t)
+            FAV_MMA_COMMITS
+            "}"
+            ::"r"(d_tmem), "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(acc), "r"(bar_a), "r"(bar_b)
+            : "memory");
+    }
+}
+#undef FAV_MMA_PV_STEP
 #undef FAV_MMA_COMMITS
 
 // commit() from a converged warp: one elected lane commits.
@@ -192,6 +225,37 @@ __device__ __forceinline__ void st_32x32b_x32(uint32_t taddr, const uint32_t (&r
           "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]),
           "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]),
           "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+
+// 32 lanes x 16 consecutive 32-bit columns.
+__device__ __forceinline__ void ld_32x32b_x16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void st_32x32b_x16(uint32_t taddr, const uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+        ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]),
+          "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]),
+          "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+}
+
+__device__ __forceinline__ void wait_ld_dep(uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.wait::ld.sync.aligned;"
+        : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+          "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]),
+          "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+        :
         : "memory");
 }
 

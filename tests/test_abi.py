@@ -88,8 +88,10 @@ def test_option_setters_validate():
     assert L.fav_set_path(-1) == 1
     assert L.fav_set_decode_splits(-1) == 1
     assert L.fav_set_decode_splits(5000) == 1
+    assert L.fav_set_prefill_grid(-1) == 1
     assert L.fav_set_path(fav.PATH_AUTO) == 0
     assert L.fav_set_decode_splits(0) == 0
+    assert L.fav_set_prefill_grid(0) == 0
 
 
 def test_python_binding_has_no_cpu_path():

@@ -15,9 +15,11 @@ pytestmark = pytest.mark.gpu
 def _reset():
     fav.set_path(fav.PATH_AUTO)
     fav.set_decode_splits(0)
+    fav.set_prefill_grid(0)
     yield
     fav.set_path(fav.PATH_AUTO)
     fav.set_decode_splits(0)
+    fav.set_prefill_grid(0)
 
 
 def W(dtype, B, Hq, Hkv, Nq, Nkv, D, causal=False, outliers=False, seed=7):
@@ -214,6 +216,28 @@ def test_prefill_bf16_v_range(D):
         tol = np.where(mag > 0, 3e-3 * np.exp2(np.ceil(np.log2(np.maximum(mag, 1e-300)))), 0.0)
         assert (np.abs(o[0, h] - ref) <= tol).all(), "head %d" % h
     assert np.abs(lse - rl).max() <= LSE_TOL
+
+
+@pytest.mark.parametrize("grid", [1, 3, 7])
+@pytest.mark.parametrize("dtype,D,causal,Hq,Hkv,N", [(I.F16, 128, True, 4, 2, 700),
+                                                     (I.BF16, 64, True, 4, 1, 520),
+                                                     (I.F16, 64, False, 2, 2, 300),
+                                                     (I.BF16, 128, False, 3, 1, 257)])
+def test_prefill_many_tiles_per_block(grid, dtype, D, causal, Hq, Hkv, N):
+    """The persistent prefill grid capped to a few blocks: each block works through many
+    query tiles of different heads and lengths in turn (score buffers, stage rings, Q buffers
+    and barrier phases carried from one tile to the next), and the results equal those of the
+    default grid bit for bit (a tile's arithmetic does not depend on which block runs it)."""
+    fav.set_path(fav.PATH_PREFILL)
+    w = W(dtype, 2, Hq, Hkv, N, N, D, causal=causal, seed=grid * 100 + D + N)
+    x = I.make_inputs(w)
+    o_ref, lse_ref = run_gpu(w, x)
+    fav.set_prefill_grid(grid)
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_PREFILL
+    check(w, o, lse, x)
+    np.testing.assert_array_equal(o, o_ref)
+    np.testing.assert_array_equal(lse, lse_ref)
 
 
 # ---- end-to-end host-buffer entry point ----
