@@ -175,6 +175,15 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *m, 
         : "memory");
 }
 
+// Prefetch of one 5-D box into L2 (no shared memory, no completion signal).
+__device__ __forceinline__ void tma_prefetch_l2_5d(const CUtensorMap *m, int x, int y, int z,
+                                                   int w, int v) {
+    asm volatile(
+        "cp.async.bulk.prefetch.tensor.5d.L2.global.tile [%0, {%1, %2, %3, %4, %5}];"
+        ::"l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(v)
+        : "memory");
+}
+
 // 5-D tiled store of one box from shared memory (bulk async-group completion).  Elements
 // outside the tensor are not written.
 __device__ __forceinline__ void tma_store_5d(const CUtensorMap *m, uint32_t src, int x, int y,

@@ -109,6 +109,7 @@ template <int D> struct PrefillCfg {
     static constexpr int kQBytes = BM * D * 2;               // one Q tile (or one O tile)
     static constexpr int kKVBytes = BN * D * 2;              // one K or V tile
     static constexpr int kUnitTab = 256;                     // units precomputed per CTA
+    static constexpr int kPrefetch = 4;                      // L2 prefetch distance (key tiles)
     // shared-memory map (offsets from the 1024-aligned base)
     static constexpr int kOffQ = 0;                          // Q buffers 0, 1 (O staging)
     static constexpr int kOffK = kOffQ + 2 * kQBytes;
@@ -202,14 +203,21 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
         return make_unit(unit_at(k));
     };
-    for (int k = threadIdx.x; k < C::kUnitTab; k += blockDim.x) {
-        const int u = unit_at(k);
-        if (u < 0) break;
-        const Unit U = make_unit(u);
-        int *e = utab + 8 * k;
-        e[0] = U.b; e[1] = U.h; e[2] = U.t; e[3] = U.n_kv; e[4] = U.kvh;
-    }
-
+    // Position in the CTA's sequence of key tiles, for the L2 prefetches that run ahead of the
+    // loads: unit index k (-1 past the end), key tile j of that unit.
+    struct TileIt {
+        int k, j;
+        Unit U;
+    };
+    auto tile_next = [&](TileIt &it) {
+        if (it.k < 0) return;
+        if (++it.j == it.U.n_kv) {
+            it.j = 0;
+            ++it.k;
+            if (unit_at(it.k) >= 0) it.U = unit(it.k);
+            else it.k = -1;
+        }
+    };
     if (warp == C::kLoadKWarp && lane == 0) {
         (void)FAV_CHECK((sbase & 1023u) == 0, status);
         (void)FAV_CHECK((sbase - raw_u32) + C::kOffTmemSlot + 4 <= fav::dynamic_smem_bytes(), status);
@@ -232,7 +240,26 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         fav::mbar_init(o_done, 1);
         for (int i = 0; i < 8; ++i) fav::mbar_init(xch_bar + 8 * i, NS * 32);
         fav::mbar_fence_init();
+        // The first Q and K tiles are requested before the rest of the set-up (unit table,
+        // TMEM allocation): they come from HBM and bound the time to the first scores.
+        fav::tma_prefetch_desc(&tmQ);
+        fav::tma_prefetch_desc(&tmK);
+        const Unit U0 = make_unit(unit_at(0));
+        fav::mbar_arrive_expect_tx(q_full, C::kQBytes);
+        fav::tma_load_5d(sQ, &tmQ, q_full, 0, U0.t * BM, 0, U0.h, U0.b);
+        for (int g = 0; g < KS && g < U0.n_kv; ++g) {
+            fav::mbar_arrive_expect_tx(k_full + 8 * g, C::kKVBytes);
+            fav::tma_load_5d(sK + g * C::kKVBytes, &tmK, k_full + 8 * g, 0, g * BN, 0, U0.kvh, U0.b);
+        }
     }
+    for (int k = threadIdx.x; k < C::kUnitTab; k += blockDim.x) {
+        const int u = unit_at(k);
+        if (u < 0) break;
+        const Unit U = make_unit(u);
+        int *e = utab + 8 * k;
+        e[0] = U.b; e[1] = U.h; e[2] = U.t; e[3] = U.n_kv; e[4] = U.kvh;
+    }
+
 #ifdef FAV_TIMING
     __shared__ long long t_ref;
     if (threadIdx.x == 0) t_ref = clock64();
@@ -253,28 +280,62 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     // (k / 2) & 1) and exchange slot k % 2, and completes o_done phase k.
     if (warp == C::kLoadKWarp) {
         // ---------------- TMA producer: Q tiles and K tiles ----------------
+        // (The stage waits poll with short suspensions: a thread suspended in a plain wait
+        // resumed several hundred cycles after the stage was released, and a K tile is needed
+        // by S about one key-tile period after its stage frees.)
         if (lane == 0) {
-            fav::tma_prefetch_desc(&tmQ);
-            fav::tma_prefetch_desc(&tmK);
+#ifdef FAV_TIMING
+            long long tsk[32];
+            for (int i = 0; i < 32; ++i) tsk[i] = 0;
+#endif
             int g = 0;
             bool ok = true;
+            // L2 prefetches run kPrefetch key tiles ahead of the loads (the ring only covers
+            // the L2 latency; a tile that misses L2 would stall S otherwise), and Q tiles a unit
+            // ahead.
+            TileIt pf{0, 0, unit(0)};
+            for (int i = 0; i < C::kPrefetch; ++i) {
+                if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                tile_next(pf);
+            }
+            const int early = min(KS, unit(0).n_kv);      // K tiles requested at the start
             for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
                 const Unit U = unit(k);
                 const int qb = k & 1;
-                // Q buffer qb was last read by unit k - 2's S MMAs
+                if (unit_at(k + 1) >= 0) {
+                    const Unit Un = unit(k + 1);
+                    fav::tma_prefetch_l2_5d(&tmQ, 0, Un.t * BM, 0, Un.h, Un.b);
+                }
+                // Q buffer qb was last read by unit k - 2's S MMAs (unit 0's Q: requested at the start)
                 if (k >= 2 && !fav::mbar_wait(q_empty + 8 * qb, ((k >> 1) - 1) & 1, status)) break;
-                fav::mbar_arrive_expect_tx(q_full + 8 * qb, C::kQBytes);
-                fav::tma_load_5d(sQ + qb * C::kQBytes, &tmQ, q_full + 8 * qb, 0, U.t * BM, 0, U.h, U.b);
+                if (k > 0) {
+                    fav::mbar_arrive_expect_tx(q_full + 8 * qb, C::kQBytes);
+                    fav::tma_load_5d(sQ + qb * C::kQBytes, &tmQ, q_full + 8 * qb, 0, U.t * BM, 0, U.h, U.b);
+                }
                 for (int j = 0; j < U.n_kv; ++j, ++g) {
                     const int st = g % KS;
-                    if (g >= KS && !fav::mbar_wait(k_empty + 8 * st, ((g / KS) - 1) & 1, status)) {
+                    if (g < early) {
+                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                        tile_next(pf);
+                        continue;
+                    }
+                    if (g >= KS && !fav::mbar_wait_fast(k_empty + 8 * st, ((g / KS) - 1) & 1, status)) {
                         ok = false;
                         break;
                     }
                     fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
                     fav::tma_load_5d(sK + st * C::kKVBytes, &tmK, k_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
+#ifdef FAV_TIMING
+                    if (g < 32) tsk[g] = clock64();
+#endif
+                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                    tile_next(pf);
                 }
             }
+#ifdef FAV_TIMING
+            if (blockIdx.x == 0)
+                for (int i = 0; i < 32; ++i) printf("[kload] G=%2d issued %6lld\n", i, tsk[i] - t_ref);
+#endif
         }
     } else if (warp == C::kLoadVWarp) {
         // ---------------- TMA producer: V tiles ----------------
@@ -282,11 +343,18 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             fav::tma_prefetch_desc(&tmV);
             int g = 0;
             bool ok = true;
+            TileIt pf{0, 0, unit(0)};
+            for (int i = 0; i < C::kPrefetch; ++i) {
+                if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                tile_next(pf);
+            }
             for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
                 const Unit U = unit(k);
                 for (int j = 0; j < U.n_kv; ++j, ++g) {
                     const int st = g % VS;
-                    if (g >= VS && !fav::mbar_wait(v_empty + 8 * st, ((g / VS) - 1) & 1, status)) {
+                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                    tile_next(pf);
+                    if (g >= VS && !fav::mbar_wait_fast(v_empty + 8 * st, ((g / VS) - 1) & 1, status)) {
                         ok = false;
                         break;
                     }
@@ -329,7 +397,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             return __all_sync(0xffffffffu, fav::mbar_wait(bar, parity, status)) != 0;
         };
 #ifdef FAV_TIMING
-        __shared__ long long tsm[32][4];
+        __shared__ long long tsm[32][6];
         const long long t_start = t_ref;
 #define FAV_TSM(g, c) do { if ((g) < 32 && lane == 0) tsm[g][c] = clock64(); } while (0)
 #else
@@ -347,6 +415,16 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             if (js == 0 && !wait_all(q_full + 8 * (ks & 1), (ks >> 1) & 1)) return false;
             return wait_all(k_full + 8 * (Gs % KS), (Gs / KS) & 1);
         };
+        // after S(Gs) has been issued: the Q buffer is released with the unit's last S
+        auto advance_s = [&]() {
+            if (js + 1 == Us.n_kv) fav::tc::commit_elect(q_empty + 8 * (ks & 1));
+            ++Gs;
+            if (++js == Us.n_kv) {
+                js = 0;
+                us = unit_at(++ks);
+                if (us >= 0) Us = unit(ks);
+            }
+        };
         auto issue_next_s = [&]() {
             if (us < 0) return;                      // no further tile
             const int qb = ks & 1, st = Gs % KS;
@@ -354,13 +432,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 tmem + C::colS(Gs & 1), dq0 + (uint64_t)((qb * C::kQBytes) >> 4),
                 dk0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_qk, 0u, s_full + 8 * (Gs & 1),
                 k_empty + 8 * st);
-            if (js + 1 == Us.n_kv) fav::tc::commit_elect(q_empty + 8 * qb);   // unit's last S
-            ++Gs;
-            if (++js == Us.n_kv) {
-                js = 0;
-                us = unit_at(++ks);
-                if (us >= 0) Us = unit(ks);
-            }
+            advance_s();
         };
         bool ok = wait_next_s();
         if (ok) {
@@ -376,15 +448,33 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         // placed right after a burst overlaps the MMAs still queued, while one placed before a
         // burst that the pipe is waiting for leaves it idle.  Per key tile G: the weights,
         // P(G).V, then (behind it) K(G+2) / Q and V(G+1), then S(G+2).
+        // Per key tile G the tensor core needs the weights P(G) and V(G) for P(G).V, then K(G+2)
+        // (and the Q tile of its unit) for S(G+2).  A barrier test costs 100-200 cycles while the
+        // MMAs and TMA copies keep shared memory busy, and the issuing lane blocks until the pipe
+        // has taken most of a burst, so tests placed between bursts leave the pipe idle.  All the
+        // barriers of a tile are therefore tested at once, one per lane (a single shared-memory
+        // instruction), and both bursts follow back to back; if one is not ready the warp waits
+        // for each in turn instead.
         int Gp = 0;
-        if (ok) ok = wait_all(v_full, 0);            // V(0)
         for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
             const Unit U = unit(k);
-            const bool more_units = unit_at(k + 1) >= 0;
             for (int j = 0; j < U.n_kv; ++j, ++Gp) {
                 const int vs = Gp % VS;
                 FAV_TSM(Gp, 0);
-                if (!(ok = wait_all(p_full + 8 * (Gp & 1), (Gp >> 1) & 1))) break;
+                // lane 0: P(G); lane 1: V(G)
+                uint32_t tb = p_full + 8 * (Gp & 1), tp = (Gp >> 1) & 1;
+                if (lane == 1) { tb = v_full + 8 * vs; tp = (Gp / VS) & 1; }
+                const bool ready_pv = fav::mbar_test(tb, tp);
+#ifdef FAV_TIMING
+                {
+                    const unsigned nb = __ballot_sync(0xffffffffu, !ready_pv) & 0x3u;
+                    if (Gp < 32 && lane == 0) tsm[Gp][4] = nb;
+                }
+#endif
+                if (!__all_sync(0xffffffffu, ready_pv)) {
+                    if (!(ok = wait_all(p_full + 8 * (Gp & 1), (Gp >> 1) & 1))) break;
+                    if (!(ok = wait_all(v_full + 8 * vs, (Gp / VS) & 1))) break;
+                }
                 FAV_TSM(Gp, 1);
                 fav::tc::fence_after();
                 fav::tc::mma_pv_split<NS>(tmem + C::kColO, tmem + C::colS(Gp & 1),
@@ -392,12 +482,21 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                                           j > 0 ? 1u : 0u, v_empty + 8 * vs, pv_done);
                 if (j + 1 == U.n_kv) fav::tc::commit_elect(o_done);   // the unit's O is final
                 FAV_TSM(Gp, 2);
-                if (!(ok = wait_next_s())) break;
-                if (j + 1 < U.n_kv || more_units) {
-                    const int g1 = Gp + 1;
-                    if (!(ok = wait_all(v_full + 8 * (g1 % VS), (g1 / VS) & 1))) break;
+                // behind the queued P.V MMAs: lane 0: K(G+2); lane 1: the Q tile of its unit
+                if (us >= 0) {
+                    uint32_t kb = k_full + 8 * (Gs % KS), kp = (Gs / KS) & 1;
+                    if (js == 0 && lane == 1) { kb = q_full + 8 * (ks & 1); kp = (ks >> 1) & 1; }
+                    const bool ready_s = fav::mbar_test(kb, kp);
+#ifdef FAV_TIMING
+                    {
+                        const unsigned nb = __ballot_sync(0xffffffffu, !ready_s) & 0x3u;
+                        if (Gp < 32 && lane == 0) tsm[Gp][4] |= nb << 2;
+                    }
+#endif
+                    if (!__all_sync(0xffffffffu, ready_s) && !(ok = wait_next_s())) break;
+                    fav::tc::fence_after();
                 }
-                fav::tc::fence_after();
+                FAV_TSM(Gp, 5);
                 issue_next_s();
                 FAV_TSM(Gp, 3);
             }
@@ -405,8 +504,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
 #ifdef FAV_TIMING
         if (blockIdx.x == 0 && lane == 0)
             for (int g = 0; g < min(Gp, 32); ++g)
-                printf("[mma] G=%2d start %6lld got_p %6lld pv_issued %6lld s_issued %6lld\n", g,
-                       tsm[g][0] - t_start, tsm[g][1] - t_start, tsm[g][2] - t_start, tsm[g][3] - t_start);
+                printf("[mma] G=%2d start %6lld got_p %6lld pv_issued %6lld notready(p,v,k,q) %x s_ready %6lld s_issued %6lld\n", g,
+                       tsm[g][0] - t_start, tsm[g][1] - t_start, tsm[g][2] - t_start, (unsigned)tsm[g][4],
+                       tsm[g][5] - t_start, tsm[g][3] - t_start);
 #endif
 #undef FAV_TSM
     } else {

@@ -189,6 +189,7 @@ __device__ __forceinline__ void mma_pv_split(uint32_t d_tmem, uint32_t a_tmem, u
             : "memory");
     }
 }
+
 #undef FAV_MMA_PV_STEP
 #undef FAV_MMA_COMMITS
 
