@@ -139,6 +139,32 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int *st
     return mbar_wait_slow(bar, parity, status);
 }
 
+// The same bounded waits with the slow path inlined, for kernels whose warp roles run under
+// setmaxnreg register budgets (a call to an out-of-line function cannot be register-allocated
+// inside such a role).
+__device__ __forceinline__ bool mbar_wait_il(uint32_t bar, uint32_t parity, int *status) {
+    if (mbar_try(bar, parity)) return true;
+    const uint64_t t0 = globaltimer();
+    while (true) {
+        if (mbar_try(bar, parity)) return true;
+        if (globaltimer() - t0 > FAV_WAIT_NS) {
+            atomicExch(status, 5);
+            return false;
+        }
+    }
+}
+__device__ __forceinline__ bool mbar_wait_fast_il(uint32_t bar, uint32_t parity, int *status) {
+    if (mbar_try_hint(bar, parity, 20)) return true;
+    const uint64_t t0 = globaltimer();
+    while (true) {
+        if (mbar_try_hint(bar, parity, 20)) return true;
+        if (globaltimer() - t0 > FAV_WAIT_NS) {
+            atomicExch(status, 5);
+            return false;
+        }
+    }
+}
+
 // ---- TMA ------------------------------------------------------------------------------
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *m) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
@@ -204,6 +230,16 @@ __device__ __forceinline__ void bulk_wait_read_all() {
 // Waits until this thread's committed bulk stores have completed.
 __device__ __forceinline__ void bulk_wait_all() {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// ---- per-warpgroup register budgets ----
+// Executed by all four warps of a warpgroup: release registers to (dec) or take them from (inc)
+// the pool the block was launched with.
+template <uint32_t N> __device__ __forceinline__ void setmaxnreg_inc() {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N> __device__ __forceinline__ void setmaxnreg_dec() {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
 
 // ---- named barriers (subsets of warps) --------------------------------------------------

@@ -23,19 +23,23 @@
 //     O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, M = max_s m_s.
 //     The point of the split: a tile's softmax runs on eight warps (two per scheduler) with no
 //     exchange between them, and takes about as long as the tile's MMAs.
-//   * the merged O tile is written into the unit's (by then free) Q buffer and stored with
-//     one TMA tensor store.
+//   * an epilogue warpgroup merges the splits once the unit's last P.V has completed, writes
+//     the O tile into the unit's (by then free) Q buffer, and one TMA tensor store writes it
+//     out; the softmax warps go on with the next unit meanwhile, and the next unit's first P.V
+//     (which overwrites O_0 and O_1) waits only until the epilogue has read them.
 // TMEM (512 columns): score buffers 0 | 1 (128 columns each; the fp16 weights of split s
 // overwrite the first half of its own score columns), then O_0 | O_1.
 // The running maximum is updated lazily: O_s and l_s are rescaled only when the maximum grows
 // by more than 2^4 (log2 domain); the weights are stored as p * 2^11 (below 2^15, inside
 // fp16's range).  O_s / l_s keeps the same maximum as its weights, so the result is unchanged.
 //
-// Warp roles (384 threads): warps 0-7 softmax (TMEM lane quarter = warp % 4, key split =
-// warp / 4; one thread per query row and split); warp 8 = TMEM owner + MMA issuer (the whole
-// warp, one elected lane issuing each burst and committing the barrier arrivals inside the
-// same asm block); warp 9 = Q/K producer, warp 10 = V producer (two issuing warps keep more TMA
-// copies in flight than one); warp 11 = O stores.
+// Warp roles (512 threads, four warpgroups with their own register budgets, setmaxnreg):
+// warps 0-7 softmax (TMEM lane quarter = warp % 4, key split = warp / 4; one thread per query
+// row and split; 176 registers); warp 8 = TMEM owner + MMA issuer (the whole warp, one elected
+// lane issuing each burst and committing the barrier arrivals inside the same asm block);
+// warp 9 = Q/K producer, warp 10 = V producer (two issuing warps keep more TMA copies in
+// flight than one); warp 11 = O stores (warps 8-11: 56 registers); warps 12-15 = epilogue (one
+// thread per query row; 96 registers).
 //
 // Issue order of the tensor core, per CTA over the global sequence G of key tiles (all units):
 //   S(0), S(1), P(0).V, S(2), P(1).V, S(3), ...    S(G) into score buffer G % 2
@@ -103,7 +107,14 @@ template <int D> struct PrefillCfg {
     static constexpr int kLoadKWarp = kSoftWarps + 1;        // Q and K
     static constexpr int kLoadVWarp = kSoftWarps + 2;
     static constexpr int kStoreWarp = kSoftWarps + 3;        // O tiles (TMA store)
-    static constexpr int kThreads = 32 * (kSoftWarps + 4);
+    static constexpr int kEpiWarp0 = kSoftWarps + 4;         // epilogue warpgroup (4 warps)
+    static constexpr int kThreads = 32 * (kSoftWarps + 8);
+    // Register budgets per warpgroup (setmaxnreg; launched with 65536 / kThreads = 128 each):
+    // softmax 176, MMA / producers / store 56, epilogue 96.  Sum 2*128*176 + 128*56 + 128*96 =
+    // 64512 <= 65536, and per scheduler (one warp of each warpgroup) 32 * 504 <= 16384.
+    static constexpr int kRegSoftmax = 176, kRegIssue = 56, kRegEpi = 96;
+    static constexpr int kRegLaunch = 65536 / kThreads;       // every warpgroup at the join
+    static_assert(2 * 128 * kRegSoftmax + 128 * kRegIssue + 128 * kRegEpi <= 65536, "registers");
     static constexpr int kKStages = 2;                       // K ring depth
     static constexpr int kVStages = 2;                       // V ring depth
     static constexpr int kQBytes = BM * D * 2;               // one Q tile (or one O tile)
@@ -118,7 +129,7 @@ template <int D> struct PrefillCfg {
     static constexpr int kXchBytes = 2 * 4 * kSplits * 32 * 8;
     static constexpr int kOffUnits = kOffXch + kXchBytes;         // int[kUnitTab][8]
     static constexpr int kOffBar = kOffUnits + kUnitTab * 32;
-    static constexpr int kNumBars = 2 + 2 + 2 * kKStages + 2 * kVStages + 2 + 2 + 2 + 8 + 2;
+    static constexpr int kNumBars = 2 + 2 + 2 * kKStages + 2 * kVStages + 2 + 2 + 2 + 2 + 2 + 1;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
     static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
     static constexpr uint32_t kTmemCols = 512;
@@ -157,8 +168,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     const uint32_t p_full = s_full + 16;          // [2] per score buffer (weights stored)
     const uint32_t pv_done = p_full + 16;         // P(G).V completed, once per key tile
     const uint32_t o_done = pv_done + 8;          // a unit's last P.V completed, once per unit
-    const uint32_t xch_bar = o_done + 8;          // [2][4] split (m, l) exchange per quarter
-    const uint32_t o_staged = xch_bar + 64;       // [2] O tile written into Q buffer k % 2
+    const uint32_t xch_bar = o_done + 8;          // [2] (m, l) of every row and split written
+    const uint32_t o_staged = xch_bar + 16;       // [2] O tile written into Q buffer k % 2
+    const uint32_t o_free = o_staged + 16;        // the epilogue has read the unit's O
     float2 *xch = reinterpret_cast<float2 *>(smem + C::kOffXch);
     int *utab = reinterpret_cast<int *>(smem + C::kOffUnits);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffTmemSlot);
@@ -224,7 +236,8 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         for (int i = 0; i < 2; ++i) {
             fav::mbar_init(q_full + 8 * i, 1);
             fav::mbar_init(q_empty + 8 * i, 2);          // last S commit + O store read
-            fav::mbar_init(o_staged + 8 * i, C::kSoftWarps * 32);
+            fav::mbar_init(o_staged + 8 * i, 128);          // epilogue threads
+            fav::mbar_init(xch_bar + 8 * i, C::kSoftWarps * 32);
             fav::mbar_init(s_full + 8 * i, 1);
             fav::mbar_init(p_full + 8 * i, C::kSoftWarps);
         }
@@ -238,7 +251,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
         fav::mbar_init(pv_done, 1);
         fav::mbar_init(o_done, 1);
-        for (int i = 0; i < 8; ++i) fav::mbar_init(xch_bar + 8 * i, NS * 32);
+        fav::mbar_init(o_free, 128);
         fav::mbar_fence_init();
         // The first Q and K tiles are requested before the rest of the set-up (unit table,
         // TMEM allocation): they come from HBM and bound the time to the first scores.
@@ -278,239 +291,10 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     // (parity (G / KS) & 1), V stage G % VS, score buffer G % 2 (s_full / p_full parity
     // (G / 2) & 1) and completes pv_done phase G; unit k uses Q buffer k % 2 (parity
     // (k / 2) & 1) and exchange slot k % 2, and completes o_done phase k.
-    if (warp == C::kLoadKWarp) {
-        // ---------------- TMA producer: Q tiles and K tiles ----------------
-        // (The stage waits poll with short suspensions: a thread suspended in a plain wait
-        // resumed several hundred cycles after the stage was released, and a K tile is needed
-        // by S about one key-tile period after its stage frees.)
-        if (lane == 0) {
-#ifdef FAV_TIMING
-            long long tsk[32];
-            for (int i = 0; i < 32; ++i) tsk[i] = 0;
-#endif
-            int g = 0;
-            bool ok = true;
-            // L2 prefetches run kPrefetch key tiles ahead of the loads (the ring only covers
-            // the L2 latency; a tile that misses L2 would stall S otherwise), and Q tiles a unit
-            // ahead.
-            TileIt pf{0, 0, unit(0)};
-            for (int i = 0; i < C::kPrefetch; ++i) {
-                if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                tile_next(pf);
-            }
-            const int early = min(KS, unit(0).n_kv);      // K tiles requested at the start
-            for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
-                const Unit U = unit(k);
-                const int qb = k & 1;
-                if (unit_at(k + 1) >= 0) {
-                    const Unit Un = unit(k + 1);
-                    fav::tma_prefetch_l2_5d(&tmQ, 0, Un.t * BM, 0, Un.h, Un.b);
-                }
-                // Q buffer qb was last read by unit k - 2's S MMAs (unit 0's Q: requested at the start)
-                if (k >= 2 && !fav::mbar_wait(q_empty + 8 * qb, ((k >> 1) - 1) & 1, status)) break;
-                if (k > 0) {
-                    fav::mbar_arrive_expect_tx(q_full + 8 * qb, C::kQBytes);
-                    fav::tma_load_5d(sQ + qb * C::kQBytes, &tmQ, q_full + 8 * qb, 0, U.t * BM, 0, U.h, U.b);
-                }
-                for (int j = 0; j < U.n_kv; ++j, ++g) {
-                    const int st = g % KS;
-                    if (g < early) {
-                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                        tile_next(pf);
-                        continue;
-                    }
-                    if (g >= KS && !fav::mbar_wait_fast(k_empty + 8 * st, ((g / KS) - 1) & 1, status)) {
-                        ok = false;
-                        break;
-                    }
-                    fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
-                    fav::tma_load_5d(sK + st * C::kKVBytes, &tmK, k_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
-#ifdef FAV_TIMING
-                    if (g < 32) tsk[g] = clock64();
-#endif
-                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                    tile_next(pf);
-                }
-            }
-#ifdef FAV_TIMING
-            if (blockIdx.x == 0)
-                for (int i = 0; i < 32; ++i) printf("[kload] G=%2d issued %6lld\n", i, tsk[i] - t_ref);
-#endif
-        }
-    } else if (warp == C::kLoadVWarp) {
-        // ---------------- TMA producer: V tiles ----------------
-        if (lane == 0) {
-            fav::tma_prefetch_desc(&tmV);
-            int g = 0;
-            bool ok = true;
-            TileIt pf{0, 0, unit(0)};
-            for (int i = 0; i < C::kPrefetch; ++i) {
-                if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                tile_next(pf);
-            }
-            for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
-                const Unit U = unit(k);
-                for (int j = 0; j < U.n_kv; ++j, ++g) {
-                    const int st = g % VS;
-                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                    tile_next(pf);
-                    if (g >= VS && !fav::mbar_wait_fast(v_empty + 8 * st, ((g / VS) - 1) & 1, status)) {
-                        ok = false;
-                        break;
-                    }
-                    fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
-                    fav::tma_load_5d(sV + st * C::kKVBytes, &tmV, v_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
-                }
-            }
-        }
-    } else if (warp == C::kStoreWarp) {
-        // ---------------- O tiles: one TMA store per unit from its (free) Q buffer ----------------
-        if (lane == 0) {
-            fav::tma_prefetch_desc(&tmO);
-            for (int k = 0, u; (u = unit_at(k)) >= 0; ++k) {
-                const Unit U = unit(k);
-                const int qb = k & 1;
-                if (!fav::mbar_wait(o_staged + 8 * qb, (k >> 1) & 1, status)) break;
-                fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.t * BM, 0, U.h, U.b);
-                fav::bulk_commit_group();
-                fav::bulk_wait_read_all();         // the buffer may take the next Q tile
-                fav::mbar_arrive(q_empty + 8 * qb);
-            }
-            fav::bulk_wait_all();
-        }
-    } else if (warp == C::kMmaWarp) {
-        // ---------------- MMA issuer: the whole warp, converged; one elected lane issues ----------------
-        constexpr bool bf = IsBF16<T>::value;
-        constexpr uint32_t idesc_qk = fav::tc::idesc_f16(BM, BN, bf, false);
-        constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, false, true);      // fp16 P, V
-        // Base descriptors are built once; a tile only adds its byte offset (>> 4) to the
-        // start-address field, which cannot carry out of its 14 bits (addresses < 256 KB).
-        const uint64_t dq0 = fav::tc::sdesc_sw128(sQ, 16, 1024);
-        const uint64_t dk0 = fav::tc::sdesc_sw128(sK, 16, 1024);
-        const uint64_t dv0 = fav::tc::sdesc_sw128(sV, BN * 128, 1024);
-        // Every lane waits; the outcome is made warp-uniform so that a bounded wait that gives
-        // up takes the whole warp out of the loop together (the bursts' elect.sync needs all
-        // 32 lanes).
-        // (A non-blocking test first: most of these phases have completed long before.)
-        auto wait_all = [&](uint32_t bar, uint32_t parity) -> bool {
-            if (__all_sync(0xffffffffu, fav::mbar_test(bar, parity))) return true;
-            return __all_sync(0xffffffffu, fav::mbar_wait(bar, parity, status)) != 0;
-        };
-#ifdef FAV_TIMING
-        __shared__ long long tsm[32][6];
-        const long long t_start = t_ref;
-#define FAV_TSM(g, c) do { if ((g) < 32 && lane == 0) tsm[g][c] = clock64(); } while (0)
-#else
-#define FAV_TSM(g, c) do { } while (0)
-#endif
-        // Scores run two key tiles ahead of the P.V products: (ks, js) is the next tile whose
-        // S is due, Gs its position in the CTA's sequence.
-        int ks = 0, js = 0, Gs = 0;
-        int us = unit_at(0);
-        Unit Us;
-        if (us >= 0) Us = unit(0);
-        // operands of the next S ready (Q of its unit, its K tile)?
-        auto wait_next_s = [&]() -> bool {
-            if (us < 0) return true;
-            if (js == 0 && !wait_all(q_full + 8 * (ks & 1), (ks >> 1) & 1)) return false;
-            return wait_all(k_full + 8 * (Gs % KS), (Gs / KS) & 1);
-        };
-        // after S(Gs) has been issued: the Q buffer is released with the unit's last S
-        auto advance_s = [&]() {
-            if (js + 1 == Us.n_kv) fav::tc::commit_elect(q_empty + 8 * (ks & 1));
-            ++Gs;
-            if (++js == Us.n_kv) {
-                js = 0;
-                us = unit_at(++ks);
-                if (us >= 0) Us = unit(ks);
-            }
-        };
-        auto issue_next_s = [&]() {
-            if (us < 0) return;                      // no further tile
-            const int qb = ks & 1, st = Gs % KS;
-            fav::tc::mma_ss_burst_k128<D / 16>(
-                tmem + C::colS(Gs & 1), dq0 + (uint64_t)((qb * C::kQBytes) >> 4),
-                dk0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_qk, 0u, s_full + 8 * (Gs & 1),
-                k_empty + 8 * st);
-            advance_s();
-        };
-        bool ok = wait_next_s();
-        if (ok) {
-            fav::tc::fence_after();
-            issue_next_s();
-            ok = wait_next_s();
-            if (ok) {
-                fav::tc::fence_after();
-                issue_next_s();
-            }
-        }
-        // The issuing lane blocks until the tensor pipe has taken most of a burst, so a wait
-        // placed right after a burst overlaps the MMAs still queued, while one placed before a
-        // burst that the pipe is waiting for leaves it idle.  Per key tile G: the weights,
-        // P(G).V, then (behind it) K(G+2) / Q and V(G+1), then S(G+2).
-        // Per key tile G the tensor core needs the weights P(G) and V(G) for P(G).V, then K(G+2)
-        // (and the Q tile of its unit) for S(G+2).  A barrier test costs 100-200 cycles while the
-        // MMAs and TMA copies keep shared memory busy, and the issuing lane blocks until the pipe
-        // has taken most of a burst, so tests placed between bursts leave the pipe idle.  All the
-        // barriers of a tile are therefore tested at once, one per lane (a single shared-memory
-        // instruction), and both bursts follow back to back; if one is not ready the warp waits
-        // for each in turn instead.
-        int Gp = 0;
-        for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
-            const Unit U = unit(k);
-            for (int j = 0; j < U.n_kv; ++j, ++Gp) {
-                const int vs = Gp % VS;
-                FAV_TSM(Gp, 0);
-                // lane 0: P(G); lane 1: V(G)
-                uint32_t tb = p_full + 8 * (Gp & 1), tp = (Gp >> 1) & 1;
-                if (lane == 1) { tb = v_full + 8 * vs; tp = (Gp / VS) & 1; }
-                const bool ready_pv = fav::mbar_test(tb, tp);
-#ifdef FAV_TIMING
-                {
-                    const unsigned nb = __ballot_sync(0xffffffffu, !ready_pv) & 0x3u;
-                    if (Gp < 32 && lane == 0) tsm[Gp][4] = nb;
-                }
-#endif
-                if (!__all_sync(0xffffffffu, ready_pv)) {
-                    if (!(ok = wait_all(p_full + 8 * (Gp & 1), (Gp >> 1) & 1))) break;
-                    if (!(ok = wait_all(v_full + 8 * vs, (Gp / VS) & 1))) break;
-                }
-                FAV_TSM(Gp, 1);
-                fav::tc::fence_after();
-                fav::tc::mma_pv_split<NS>(tmem + C::kColO, tmem + C::colS(Gp & 1),
-                                          dv0 + (uint64_t)((vs * C::kKVBytes) >> 4), idesc_pv,
-                                          j > 0 ? 1u : 0u, v_empty + 8 * vs, pv_done);
-                if (j + 1 == U.n_kv) fav::tc::commit_elect(o_done);   // the unit's O is final
-                FAV_TSM(Gp, 2);
-                // behind the queued P.V MMAs: lane 0: K(G+2); lane 1: the Q tile of its unit
-                if (us >= 0) {
-                    uint32_t kb = k_full + 8 * (Gs % KS), kp = (Gs / KS) & 1;
-                    if (js == 0 && lane == 1) { kb = q_full + 8 * (ks & 1); kp = (ks >> 1) & 1; }
-                    const bool ready_s = fav::mbar_test(kb, kp);
-#ifdef FAV_TIMING
-                    {
-                        const unsigned nb = __ballot_sync(0xffffffffu, !ready_s) & 0x3u;
-                        if (Gp < 32 && lane == 0) tsm[Gp][4] |= nb << 2;
-                    }
-#endif
-                    if (!__all_sync(0xffffffffu, ready_s) && !(ok = wait_next_s())) break;
-                    fav::tc::fence_after();
-                }
-                FAV_TSM(Gp, 5);
-                issue_next_s();
-                FAV_TSM(Gp, 3);
-            }
-        }
-#ifdef FAV_TIMING
-        if (blockIdx.x == 0 && lane == 0)
-            for (int g = 0; g < min(Gp, 32); ++g)
-                printf("[mma] G=%2d start %6lld got_p %6lld pv_issued %6lld notready(p,v,k,q) %x s_ready %6lld s_issued %6lld\n", g,
-                       tsm[g][0] - t_start, tsm[g][1] - t_start, tsm[g][2] - t_start, (unsigned)tsm[g][4],
-                       tsm[g][5] - t_start, tsm[g][3] - t_start);
-#endif
-#undef FAV_TSM
-    } else {
-        // ---------------- softmax / correction / epilogue: one thread per query row and split ----------------
+    // Roles by warpgroup; each branch opens with its register budget (setmaxnreg).
+    if (warp < C::kSoftWarps) {
+        fav::setmaxnreg_inc<C::kRegSoftmax>();
+        // ---------------- softmax / correction: one thread per query row and split ----------------
         const int quarter = warp & 3, split = warp >> 2;
         const int row = quarter * 32 + lane;
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
@@ -519,93 +303,11 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         bool ok = true;
 #ifdef FAV_TIMING
         long long ts[32][5];
-        long long te[8], te1[8], te2[8], te3[8];
         const long long t_start = t_ref;
 #define FAV_TSS(c) do { if (Gt < 32) ts[Gt][c] = clock64(); } while (0)
 #else
 #define FAV_TSS(c) do { } while (0)
 #endif
-        // Epilogue of unit kk (running maximum m, sum l of this row and split): merge the
-        // splits, O / L, LSE.  It runs after the next unit's first weights are stored (so that
-        // the wait for the unit's last P.V overlaps that softmax) and before they are released
-        // (the next unit's first P.V overwrites every O_s).
-        auto epilogue = [&](const Unit &U, float m, float l, int kk) -> bool {
-            if (!__all_sync(~0u, fav::mbar_wait(o_done, kk & 1, status))) return false;
-#ifdef FAV_TIMING
-            if (kk < 8) te1[kk] = clock64();
-#endif
-            fav::tc::fence_after();
-            // (m_s, l_s) of this row's splits through shared memory (slot kk % 2)
-            const int xs = kk & 1;
-            float2 *xrow = xch + ((xs * 4 + quarter) * NS) * 32 + lane;
-            xrow[split * 32] = make_float2(m, l);
-            fav::mbar_arrive(xch_bar + 8 * (xs * 4 + quarter));
-            if (!__all_sync(~0u, fav::mbar_wait(xch_bar + 8 * (xs * 4 + quarter), (kk >> 1) & 1, status)))
-                return false;
-#ifdef FAV_TIMING
-            if (kk < 8) te2[kk] = clock64();
-#endif
-            float Mx = -INFINITY;
-            float2 ml[NS];
-#pragma unroll
-            for (int t = 0; t < NS; ++t) {
-                ml[t] = xrow[t * 32];
-                Mx = fmaxf(Mx, ml[t].x);
-            }
-            float w[NS], L = 0.f;
-#pragma unroll
-            for (int t = 0; t < NS; ++t) {
-                w[t] = (ml[t].x == -INFINITY) ? 0.f : fav::fast_exp2(ml[t].x - Mx);
-                L += w[t] * ml[t].y;
-            }
-            const int qi = U.t * BM + row;
-            const float vsc = kV16 ? v_scale[U.b * Hkv + U.kvh] : 1.f;   // V = v_scale * (fp16 copy)
-            const float inv_l = vsc / L;
-            // This warp's columns [split * 64, split * 64 + 64) of O -- one 64-column block of
-            // the tile -- go to the unit's Q buffer (free: the unit's S products have completed)
-            // in the TMA box layout (rows of 128 bytes, 16-byte chunks XOR-swizzled by row % 8);
-            // the store warp writes the tile out with one TMA store (rows beyond Nq are not
-            // written).
-            const uint32_t stage = sQ + (kk & 1) * C::kQBytes + split * (BM * 128) + row * 128;
-#ifdef FAV_TIMING
-            if (kk < 8) te3[kk] = clock64();
-#endif
-#pragma unroll
-            for (int c = 0; c < 2; ++c) {
-                static_assert(NS == 2, "two accumulators per chunk");
-                uint32_t v0[32], v1[32];
-                fav::tc::ld_32x32b_x32(trow + C::kColO + split * 64 + c * 32, v0);
-                fav::tc::ld_32x32b_x32(trow + C::kColO + D + split * 64 + c * 32, v1);
-                fav::tc::wait_ld_dep(v0);
-                fav::tc::wait_ld_dep(v1);
-                float acc[32];
-#pragma unroll
-                for (int e = 0; e < 32; ++e)
-                    acc[e] = fmaf(w[0], __uint_as_float(v0[e]), w[1] * __uint_as_float(v1[e]));
-#pragma unroll
-                for (int e = 0; e < 32; e += 8) {
-                    const uint32_t x0 = fav::Elem<T>::pack(acc[e] * inv_l, acc[e + 1] * inv_l);
-                    const uint32_t x1 = fav::Elem<T>::pack(acc[e + 2] * inv_l, acc[e + 3] * inv_l);
-                    const uint32_t x2 = fav::Elem<T>::pack(acc[e + 4] * inv_l, acc[e + 5] * inv_l);
-                    const uint32_t x3 = fav::Elem<T>::pack(acc[e + 6] * inv_l, acc[e + 7] * inv_l);
-                    const uint32_t chunk = (uint32_t)(c * 4 + e / 8) ^ (uint32_t)(row & 7);
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};"
-                                 ::"r"(stage + (chunk << 4)), "r"(x0), "r"(x1), "r"(x2), "r"(x3)
-                                 : "memory");
-                }
-            }
-            fav::tc::fence_proxy_async_smem();   // visible to the TMA store (async proxy)
-            fav::mbar_arrive(o_staged + 8 * (kk & 1));
-            if (split == 0 && qi < Nq && lse)
-                lse[(long long)(U.b * Hq + U.h) * Nq + qi] = (Mx - kPShift + log2f(L)) * kLn2;
-#ifdef FAV_TIMING
-            if (kk < 8) te[kk] = clock64();
-#endif
-            return true;
-        };
-        int k_pend = -1;           // unit whose epilogue is still due
-        Unit U_pend;
-        float m_pend = 0.f, l_pend = 0.f;
         for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
             const Unit U = unit(k);
             const int q0 = U.t * BM;
@@ -615,7 +317,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             float m = -INFINITY, l = 0.f;
             for (int j = 0; j < U.n_kv; ++j, ++Gt) {
                 FAV_TSS(0);
-                if (!__all_sync(~0u, fav::mbar_wait(s_full + 8 * (Gt & 1), (Gt >> 1) & 1, status))) {
+                if (!__all_sync(~0u, fav::mbar_wait_il(s_full + 8 * (Gt & 1), (Gt >> 1) & 1, status))) {
                     ok = false;
                     break;
                 }
@@ -693,7 +395,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 // G-2 and cannot have completed G (that needs these weights): the parity of phase
                 // G-1 is unambiguous.
                 if (__any_sync(~0u, rescale)) {
-                    if (!__all_sync(~0u, fav::mbar_wait(pv_done, (Gt - 1) & 1, status))) {
+                    if (!__all_sync(~0u, fav::mbar_wait_il(pv_done, (Gt - 1) & 1, status))) {
                         ok = false;
                         break;
                     }
@@ -714,14 +416,6 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                         fav::tc::st_32x32b_x32(trow + col, v);
                     }
                 }
-                // the previous unit's epilogue, between this unit's first weights and their release
-                if (j == 0 && k_pend >= 0) {
-                    if (!epilogue(U_pend, m_pend, l_pend, k_pend)) {
-                        ok = false;
-                        break;
-                    }
-                    k_pend = -1;
-                }
                 fav::tc::wait_st();
                 fav::tc::fence_before();
                 __syncwarp();
@@ -729,24 +423,319 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 FAV_TSS(4);
             }
             if (!ok) break;
-            k_pend = k;
-            U_pend = U;
-            m_pend = m;
-            l_pend = l;
+            // (m, l) of this row and split for the epilogue warpgroup (slot k % 2)
+            xch[((((k & 1) * 4 + quarter) * NS) + split) * 32 + lane] = make_float2(m, l);
+            fav::mbar_arrive(xch_bar + 8 * (k & 1));
         }
-        if (ok && k_pend >= 0) (void)epilogue(U_pend, m_pend, l_pend, k_pend);
 #ifdef FAV_TIMING
         if (blockIdx.x == 0 && (threadIdx.x & 127) == 0) {
             for (int g = 0; g < min(Gt, 32); ++g)
                 printf("[sm%d] G=%2d wait %6lld s_ready %6lld max %6lld exp %6lld arrive %6lld\n",
                        split, g, ts[g][0] - t_start, ts[g][1] - t_start, ts[g][2] - t_start,
                        ts[g][3] - t_start, ts[g][4] - t_start);
-            for (int kk = 0; kk < 3; ++kk)
-                printf("[epi%d] unit %d o_done %6lld xch %6lld merged %6lld done %6lld\n", split, kk,
-                       te1[kk] - t_start, te2[kk] - t_start, te3[kk] - t_start, te[kk] - t_start);
         }
 #endif
 #undef FAV_TSS
+        fav::setmaxnreg_dec<C::kRegLaunch>();      // back to the launch budget for the join
+    } else if (warp >= C::kEpiWarp0) {
+        fav::setmaxnreg_dec<C::kRegEpi>();
+        // ---------------- epilogue: merge the splits, O / L, LSE; one thread per query row ----------------
+        // O = (2^(m_0 - M) O_0 + 2^(m_1 - M) O_1) / L, L = 2^(m_0 - M) l_0 + 2^(m_1 - M) l_1,
+        // M = max(m_0, m_1).  The O tile goes, rounded to the I/O type, into the unit's Q buffer
+        // (free: the unit's S products have completed) in the TMA box layout (rows of 128 bytes,
+        // 16-byte chunks XOR-swizzled by row % 8); the store warp writes it out with one TMA
+        // store (rows beyond Nq are not written).  As soon as O has been read, the next unit's
+        // first P.V (which overwrites O_0 and O_1) may run.
+        const int quarter = warp & 3;
+        const int row = quarter * 32 + lane;
+        const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+        for (int k = 0, u; (u = unit_at(k)) >= 0; ++k) {
+            const Unit U = unit(k);
+            if (!__all_sync(~0u, fav::mbar_wait_il(o_done, k & 1, status))) break;
+            if (!__all_sync(~0u, fav::mbar_wait_il(xch_bar + 8 * (k & 1), (k >> 1) & 1, status))) break;
+            fav::tc::fence_after();
+            const float2 ml0 = xch[((((k & 1) * 4 + quarter) * NS) + 0) * 32 + lane];
+            const float2 ml1 = xch[((((k & 1) * 4 + quarter) * NS) + 1) * 32 + lane];
+            const float Mx = fmaxf(ml0.x, ml1.x);
+            const float w0 = (ml0.x == -INFINITY) ? 0.f : fav::fast_exp2(ml0.x - Mx);
+            const float w1 = (ml1.x == -INFINITY) ? 0.f : fav::fast_exp2(ml1.x - Mx);
+            const float L = w0 * ml0.y + w1 * ml1.y;
+            const int qi = U.t * BM + row;
+            const float vsc = kV16 ? v_scale[U.b * Hkv + U.kvh] : 1.f;   // V = v_scale * (fp16 copy)
+            const float inv_l = vsc / L;
+            const float a0 = w0 * inv_l, a1 = w1 * inv_l;
+            const uint32_t stage = sQ + (k & 1) * C::kQBytes + row * 128;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {   // 32 columns at a time, both splits in flight
+                uint32_t v0[32], v1[32];
+                fav::tc::ld_32x32b_x32(trow + C::kColO + c * 32, v0);
+                fav::tc::ld_32x32b_x32(trow + C::kColO + D + c * 32, v1);
+                fav::tc::wait_ld_dep(v0);
+                fav::tc::wait_ld_dep(v1);
+#pragma unroll
+                for (int h = 0; h < 4; ++h) {
+                    // 8 columns = one 16-byte chunk: column block c / 2, chunk 4 (c % 2) + h
+                    uint32_t x[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int i = 8 * h + 2 * e;
+                        x[e] = fav::Elem<T>::pack(
+                            fmaf(a0, __uint_as_float(v0[i]), a1 * __uint_as_float(v1[i])),
+                            fmaf(a0, __uint_as_float(v0[i + 1]), a1 * __uint_as_float(v1[i + 1])));
+                    }
+                    const uint32_t chunk = (uint32_t)(4 * (c & 1) + h) ^ (uint32_t)(row & 7);
+                    const uint32_t addr = stage + (c >> 1) * (BM * 128) + (chunk << 4);
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};"
+                                 ::"r"(addr), "r"(x[0]), "r"(x[1]), "r"(x[2]), "r"(x[3])
+                                 : "memory");
+                }
+            }
+            // O has been read: release it to the next unit's first P.V
+            fav::tc::fence_before();
+            fav::mbar_arrive(o_free);
+            fav::tc::fence_proxy_async_smem();   // visible to the TMA store (async proxy)
+            fav::mbar_arrive(o_staged + 8 * (k & 1));
+            if (qi < Nq && lse)
+                lse[(long long)(U.b * Hq + U.h) * Nq + qi] = (Mx - kPShift + log2f(L)) * kLn2;
+        }
+        fav::setmaxnreg_inc<C::kRegLaunch>();
+    } else {
+        fav::setmaxnreg_dec<C::kRegIssue>();
+        if (warp == C::kLoadKWarp) {
+            // ---------------- TMA producer: Q tiles and K tiles ----------------
+            // (The stage waits poll with short suspensions: a thread suspended in a plain wait
+            // resumed several hundred cycles after the stage was released, and a K tile is needed
+            // by S about one key-tile period after its stage frees.)
+            if (lane == 0) {
+    #ifdef FAV_TIMING
+                long long tsk[32];
+                for (int i = 0; i < 32; ++i) tsk[i] = 0;
+    #endif
+                int g = 0;
+                bool ok = true;
+                // L2 prefetches run kPrefetch key tiles ahead of the loads (the ring only covers
+                // the L2 latency; a tile that misses L2 would stall S otherwise), and Q tiles a unit
+                // ahead.
+                TileIt pf{0, 0, unit(0)};
+                for (int i = 0; i < C::kPrefetch; ++i) {
+                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                    tile_next(pf);
+                }
+                const int early = min(KS, unit(0).n_kv);      // K tiles requested at the start
+                for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
+                    const Unit U = unit(k);
+                    const int qb = k & 1;
+                    if (unit_at(k + 1) >= 0) {
+                        const Unit Un = unit(k + 1);
+                        fav::tma_prefetch_l2_5d(&tmQ, 0, Un.t * BM, 0, Un.h, Un.b);
+                    }
+                    // Q buffer qb was last read by unit k - 2's S MMAs (unit 0's Q: requested at the start)
+                    if (k >= 2 && !fav::mbar_wait_il(q_empty + 8 * qb, ((k >> 1) - 1) & 1, status)) break;
+                    if (k > 0) {
+                        fav::mbar_arrive_expect_tx(q_full + 8 * qb, C::kQBytes);
+                        fav::tma_load_5d(sQ + qb * C::kQBytes, &tmQ, q_full + 8 * qb, 0, U.t * BM, 0, U.h, U.b);
+                    }
+                    for (int j = 0; j < U.n_kv; ++j, ++g) {
+                        const int st = g % KS;
+                        if (g < early) {
+                            if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                            tile_next(pf);
+                            continue;
+                        }
+                        if (g >= KS && !fav::mbar_wait_fast_il(k_empty + 8 * st, ((g / KS) - 1) & 1, status)) {
+                            ok = false;
+                            break;
+                        }
+                        fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
+                        fav::tma_load_5d(sK + st * C::kKVBytes, &tmK, k_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
+    #ifdef FAV_TIMING
+                        if (g < 32) tsk[g] = clock64();
+    #endif
+                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                        tile_next(pf);
+                    }
+                }
+    #ifdef FAV_TIMING
+                if (blockIdx.x == 0)
+                    for (int i = 0; i < 32; ++i) printf("[kload] G=%2d issued %6lld\n", i, tsk[i] - t_ref);
+    #endif
+            }
+        } else if (warp == C::kLoadVWarp) {
+            // ---------------- TMA producer: V tiles ----------------
+            if (lane == 0) {
+                fav::tma_prefetch_desc(&tmV);
+                int g = 0;
+                bool ok = true;
+                TileIt pf{0, 0, unit(0)};
+                for (int i = 0; i < C::kPrefetch; ++i) {
+                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                    tile_next(pf);
+                }
+                for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
+                    const Unit U = unit(k);
+                    for (int j = 0; j < U.n_kv; ++j, ++g) {
+                        const int st = g % VS;
+                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                        tile_next(pf);
+                        if (g >= VS && !fav::mbar_wait_fast_il(v_empty + 8 * st, ((g / VS) - 1) & 1, status)) {
+                            ok = false;
+                            break;
+                        }
+                        fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
+                        fav::tma_load_5d(sV + st * C::kKVBytes, &tmV, v_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
+                    }
+                }
+            }
+        } else if (warp == C::kStoreWarp) {
+            // ---------------- O tiles: one TMA store per unit from its (free) Q buffer ----------------
+            if (lane == 0) {
+                fav::tma_prefetch_desc(&tmO);
+                for (int k = 0, u; (u = unit_at(k)) >= 0; ++k) {
+                    const Unit U = unit(k);
+                    const int qb = k & 1;
+                    if (!fav::mbar_wait_il(o_staged + 8 * qb, (k >> 1) & 1, status)) break;
+                    fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.t * BM, 0, U.h, U.b);
+                    fav::bulk_commit_group();
+                    fav::bulk_wait_read_all();         // the buffer may take the next Q tile
+                    fav::mbar_arrive(q_empty + 8 * qb);
+                }
+                fav::bulk_wait_all();
+            }
+        } else {
+            // ---------------- MMA issuer: the whole warp, converged; one elected lane issues ----------------
+            constexpr bool bf = IsBF16<T>::value;
+            constexpr uint32_t idesc_qk = fav::tc::idesc_f16(BM, BN, bf, false);
+            constexpr uint32_t idesc_pv = fav::tc::idesc_f16(BM, D, false, true);      // fp16 P, V
+            // Base descriptors are built once; a tile only adds its byte offset (>> 4) to the
+            // start-address field, which cannot carry out of its 14 bits (addresses < 256 KB).
+            const uint64_t dq0 = fav::tc::sdesc_sw128(sQ, 16, 1024);
+            const uint64_t dk0 = fav::tc::sdesc_sw128(sK, 16, 1024);
+            const uint64_t dv0 = fav::tc::sdesc_sw128(sV, BN * 128, 1024);
+            // Every lane waits; the outcome is made warp-uniform so that a bounded wait that gives
+            // up takes the whole warp out of the loop together (the bursts' elect.sync needs all
+            // 32 lanes).
+            // (A non-blocking test first: most of these phases have completed long before.)
+            auto wait_all = [&](uint32_t bar, uint32_t parity) -> bool {
+                if (__all_sync(0xffffffffu, fav::mbar_test(bar, parity))) return true;
+                return __all_sync(0xffffffffu, fav::mbar_wait_il(bar, parity, status)) != 0;
+            };
+    #ifdef FAV_TIMING
+            __shared__ long long tsm[32][6];
+            const long long t_start = t_ref;
+    #define FAV_TSM(g, c) do { if ((g) < 32 && lane == 0) tsm[g][c] = clock64(); } while (0)
+    #else
+    #define FAV_TSM(g, c) do { } while (0)
+    #endif
+            // Scores run two key tiles ahead of the P.V products: (ks, js) is the next tile whose
+            // S is due, Gs its position in the CTA's sequence.
+            int ks = 0, js = 0, Gs = 0;
+            int us = unit_at(0);
+            Unit Us;
+            if (us >= 0) Us = unit(0);
+            // operands of the next S ready (Q of its unit, its K tile)?
+            auto wait_next_s = [&]() -> bool {
+                if (us < 0) return true;
+                if (js == 0 && !wait_all(q_full + 8 * (ks & 1), (ks >> 1) & 1)) return false;
+                return wait_all(k_full + 8 * (Gs % KS), (Gs / KS) & 1);
+            };
+            // after S(Gs) has been issued: the Q buffer is released with the unit's last S
+            auto advance_s = [&]() {
+                if (js + 1 == Us.n_kv) fav::tc::commit_elect(q_empty + 8 * (ks & 1));
+                ++Gs;
+                if (++js == Us.n_kv) {
+                    js = 0;
+                    us = unit_at(++ks);
+                    if (us >= 0) Us = unit(ks);
+                }
+            };
+            auto issue_next_s = [&]() {
+                if (us < 0) return;                      // no further tile
+                const int qb = ks & 1, st = Gs % KS;
+                fav::tc::mma_ss_burst_k128<D / 16>(
+                    tmem + C::colS(Gs & 1), dq0 + (uint64_t)((qb * C::kQBytes) >> 4),
+                    dk0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_qk, 0u, s_full + 8 * (Gs & 1),
+                    k_empty + 8 * st);
+                advance_s();
+            };
+            bool ok = wait_next_s();
+            if (ok) {
+                fav::tc::fence_after();
+                issue_next_s();
+                ok = wait_next_s();
+                if (ok) {
+                    fav::tc::fence_after();
+                    issue_next_s();
+                }
+            }
+            // The issuing lane blocks until the tensor pipe has taken most of a burst, so a wait
+            // placed right after a burst overlaps the MMAs still queued, while one placed before a
+            // burst that the pipe is waiting for leaves it idle.  Per key tile G: the weights,
+            // P(G).V, then (behind it) K(G+2) / Q and V(G+1), then S(G+2).
+            // Per key tile G the tensor core needs the weights P(G) and V(G) for P(G).V, then K(G+2)
+            // (and the Q tile of its unit) for S(G+2).  A barrier test costs 100-200 cycles while the
+            // MMAs and TMA copies keep shared memory busy, and the issuing lane blocks until the pipe
+            // has taken most of a burst, so tests placed between bursts leave the pipe idle.  All the
+            // barriers of a tile are therefore tested at once, one per lane (a single shared-memory
+            // instruction), and both bursts follow back to back; if one is not ready the warp waits
+            // for each in turn instead.
+            int Gp = 0;
+            for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
+                const Unit U = unit(k);
+                for (int j = 0; j < U.n_kv; ++j, ++Gp) {
+                    const int vs = Gp % VS;
+                    FAV_TSM(Gp, 0);
+                    // lane 0: P(G); lane 1: V(G)
+                    uint32_t tb = p_full + 8 * (Gp & 1), tp = (Gp >> 1) & 1;
+                    if (lane == 1) { tb = v_full + 8 * vs; tp = (Gp / VS) & 1; }
+                    const bool ready_pv = fav::mbar_test(tb, tp);
+    #ifdef FAV_TIMING
+                    {
+                        const unsigned nb = __ballot_sync(0xffffffffu, !ready_pv) & 0x3u;
+                        if (Gp < 32 && lane == 0) tsm[Gp][4] = nb;
+                    }
+    #endif
+                    if (!__all_sync(0xffffffffu, ready_pv)) {
+                        if (!(ok = wait_all(p_full + 8 * (Gp & 1), (Gp >> 1) & 1))) break;
+                        if (!(ok = wait_all(v_full + 8 * vs, (Gp / VS) & 1))) break;
+                    }
+                    // a unit's first P.V overwrites O: the previous unit's O must have been read
+                    if (j == 0 && k > 0 && !(ok = wait_all(o_free, (k - 1) & 1))) break;
+                    FAV_TSM(Gp, 1);
+                    fav::tc::fence_after();
+                    fav::tc::mma_pv_split<NS>(tmem + C::kColO, tmem + C::colS(Gp & 1),
+                                              dv0 + (uint64_t)((vs * C::kKVBytes) >> 4), idesc_pv,
+                                              j > 0 ? 1u : 0u, v_empty + 8 * vs, pv_done);
+                    if (j + 1 == U.n_kv) fav::tc::commit_elect(o_done);   // the unit's O is final
+                    FAV_TSM(Gp, 2);
+                    // behind the queued P.V MMAs: lane 0: K(G+2); lane 1: the Q tile of its unit
+                    if (us >= 0) {
+                        uint32_t kb = k_full + 8 * (Gs % KS), kp = (Gs / KS) & 1;
+                        if (js == 0 && lane == 1) { kb = q_full + 8 * (ks & 1); kp = (ks >> 1) & 1; }
+                        const bool ready_s = fav::mbar_test(kb, kp);
+    #ifdef FAV_TIMING
+                        {
+                            const unsigned nb = __ballot_sync(0xffffffffu, !ready_s) & 0x3u;
+                            if (Gp < 32 && lane == 0) tsm[Gp][4] |= nb << 2;
+                        }
+    #endif
+                        if (!__all_sync(0xffffffffu, ready_s) && !(ok = wait_next_s())) break;
+                        fav::tc::fence_after();
+                    }
+                    FAV_TSM(Gp, 5);
+                    issue_next_s();
+                    FAV_TSM(Gp, 3);
+                }
+            }
+    #ifdef FAV_TIMING
+            if (blockIdx.x == 0 && lane == 0)
+                for (int g = 0; g < min(Gp, 32); ++g)
+                    printf("[mma] G=%2d start %6lld got_p %6lld pv_issued %6lld notready(p,v,k,q) %x s_ready %6lld s_issued %6lld\n", g,
+                           tsm[g][0] - t_start, tsm[g][1] - t_start, tsm[g][2] - t_start, (unsigned)tsm[g][4],
+                           tsm[g][5] - t_start, tsm[g][3] - t_start);
+    #endif
+    #undef FAV_TSM
+        }
+        fav::setmaxnreg_inc<C::kRegLaunch>();
     }
 
     fav::tc::fence_before();
