@@ -42,6 +42,8 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="fav", choices=["fav", "reference"])
     ap.add_argument("--no-extra", action="store_true", help="headline workload only")
+    ap.add_argument("--extra", default=None,
+                    help="comma-separated indices of the extra workloads to time (default: all)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle cpu_baseline")
     return ap.parse_args()
 
@@ -324,7 +326,8 @@ def fav_arm(args, dist):
     x, ms, times, nl, path = bench_workload(w, args.steps, args.warmup)
     extras = []
     if not args.no_extra:
-        for idx in EXTRA:
+        chosen = EXTRA if args.extra is None else [int(i) for i in args.extra.split(",")]
+        for idx in chosen:
             we = I.WORKLOADS[idx]
             _, mse, te, nle, pe = bench_workload(we, args.steps, args.warmup)
             if we.Nq == 1:
