@@ -118,6 +118,36 @@ FAV_API fav_status fav_forward_strided(const void *q, const void *k, const void 
                                        int causal, fav_dtype dtype, void *stream);
 
 /*
+ * fav_decode_paged -- decode (and small-Nq) attention over a PAGED key/value cache, per sequence
+ * of its own length.  (Method section: the decode stage attends one query row per head to the
+ * whole cached sequence; a serving system keeps that cache in fixed-size pages shared by many
+ * sequences, so the keys of one sequence are not contiguous.)
+ *
+ *  q, o         device, [B, Hq, Nq, D] contiguous, `dtype`, 16-byte aligned
+ *  k_cache,     device page pools, [num_pages, page_size, Hkv, D] contiguous (the heads of a
+ *  v_cache      token side by side), `dtype`, 16-byte aligned
+ *  block_table  device int32 [B, max_pages]: key n of sequence b is row n % page_size of page
+ *               block_table[b * max_pages + n / page_size].  Pages may be shared between
+ *               sequences.  Entries past a sequence's length are not read; a page id outside
+ *               [0, num_pages) reads as zeros.
+ *  seq_lens     device int32 [B]: keys of each sequence, clamped to [0, max_pages * page_size]
+ *  lse          device [B, Hq, Nq] fp32, or NULL
+ *  page_size    a power of two in [16, 65536] (else FAV_ERR_UNSUPPORTED)
+ *  causal       bottom-right aligned per sequence: query i of sequence b sees keys
+ *               j <= seq_lens[b] - Nq + i.  A query row that sees no key (seq_lens[b] = 0, or a
+ *               causal row before the start) gets O = 0 and LSE = -inf.
+ *  other arguments as fav_forward, for decode-shaped calls: fp16/bf16, D in {64, 128},
+ *  Nq * Hq / Hkv <= 64 (else FAV_ERR_UNSUPPORTED).  Arguments are validated before anything is
+ *  launched (the device arrays' contents are not); the call is asynchronous on `stream` and
+ *  uses the split-KV workspace of fav_forward (sized for max_pages * page_size keys).
+ */
+FAV_API fav_status fav_decode_paged(const void *q, const void *k_cache, const void *v_cache,
+                                    void *o, float *lse, const int *block_table,
+                                    const int *seq_lens, int B, int Hq, int Hkv, int Nq,
+                                    int max_pages, int page_size, int num_pages, int D,
+                                    float scale, int causal, fav_dtype dtype, void *stream);
+
+/*
  * fav_forward_host -- the same operation on HOST buffers (end-to-end call).
  *
  * Copies q, k, v (host, ideally pinned) to internal device buffers, computes, copies o and lse

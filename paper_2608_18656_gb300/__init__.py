@@ -7,7 +7,7 @@ CPU fallback: without the built library every call raises.
 import ctypes
 import os
 
-__all__ = ["forward", "forward_host", "Strides", "set_path", "last_path", "set_decode_splits",
+__all__ = ["forward", "forward_host", "decode_paged", "Strides", "set_path", "last_path", "set_decode_splits",
            "last_decode_splits", "set_prefill_grid", "device_status", "release_workspace", "library_path",
            "FavError", "F32", "F16", "BF16", "PATH_AUTO", "PATH_SIMT", "PATH_DECODE",
            "PATH_PREFILL"]
@@ -57,6 +57,9 @@ def lib():
         L.fav_forward_strided.argtypes = [vp, vp, vp, vp, vp, S, S, S, S, i, i, i, i, i, i,
                                           ctypes.c_float, i, i, vp]
         L.fav_forward_strided.restype = i
+        L.fav_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i, i, i,
+                                       ctypes.c_float, i, i, vp]
+        L.fav_decode_paged.restype = i
         L.fav_status_string.argtypes = [i]
         L.fav_status_string.restype = ctypes.c_char_p
         L.fav_get_last_device_status.argtypes = []
@@ -135,6 +138,50 @@ def forward(q, k, v, causal=False, scale=None, return_lse=True, out=None, lse_ou
                                            o.data_ptr(), lse_ptr, *sd, B, Hq, Hkv, Nq, Nkv, D,
                                            float(scale), int(bool(causal)), _dtype_code(q),
                                            s.cuda_stream)
+    _check(st)
+    return o, lse
+
+
+def decode_paged(q, k_cache, v_cache, block_table, seq_lens, causal=False, scale=None,
+                 return_lse=True, out=None, lse_out=None, stream=None):
+    """Decode attention over a paged cache (fav_decode_paged).
+
+    q [B,Hq,Nq,D] contiguous; k_cache / v_cache [num_pages, page_size, Hkv, D] contiguous;
+    block_table int32 [B, max_pages] and seq_lens int32 [B], all torch CUDA tensors on one
+    device.  Returns (o, lse) like forward().
+    """
+    import torch
+    for t in (q, k_cache, v_cache, block_table, seq_lens):
+        if not t.is_cuda:
+            raise ValueError("tensors must live on a CUDA device")
+        if not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+    if k_cache.dtype != q.dtype or v_cache.dtype != q.dtype:
+        raise TypeError("q and the caches must share a dtype")
+    if block_table.dtype != torch.int32 or seq_lens.dtype != torch.int32:
+        raise TypeError("block_table and seq_lens must be int32")
+    B, Hq, Nq, D = q.shape
+    num_pages, page_size, Hkv, Dk = k_cache.shape
+    if tuple(v_cache.shape) != tuple(k_cache.shape) or Dk != D:
+        raise ValueError("shape mismatch between q and the caches")
+    if block_table.dim() != 2 or block_table.shape[0] != B or tuple(seq_lens.shape) != (B,):
+        raise ValueError("block_table must be [B, max_pages] and seq_lens [B]")
+    max_pages = block_table.shape[1]
+    if scale is None:
+        import numpy as np
+        scale = float(np.float32(1.0 / np.sqrt(D)))
+    o = out if out is not None else torch.empty(q.shape, dtype=q.dtype, device=q.device)
+    lse = None
+    if return_lse:
+        lse = lse_out if lse_out is not None else torch.empty((B, Hq, Nq), device=q.device,
+                                                              dtype=torch.float32)
+    s = stream if stream is not None else torch.cuda.current_stream(q.device)
+    with torch.cuda.device(q.device):
+        st = lib().fav_decode_paged(q.data_ptr(), k_cache.data_ptr(), v_cache.data_ptr(),
+                                    o.data_ptr(), lse.data_ptr() if lse is not None else None,
+                                    block_table.data_ptr(), seq_lens.data_ptr(), B, Hq, Hkv, Nq,
+                                    max_pages, page_size, num_pages, D, float(scale),
+                                    int(bool(causal)), _dtype_code(q), s.cuda_stream)
     _check(st)
     return o, lse
 

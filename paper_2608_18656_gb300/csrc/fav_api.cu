@@ -291,6 +291,64 @@ fav_status fav_forward(const void *q, const void *k, const void *v, void *o, flo
     return forward_impl(a, static_cast<cudaStream_t>(stream));
 }
 
+fav_status fav_decode_paged(const void *q, const void *k_cache, const void *v_cache, void *o,
+                            float *lse, const int *block_table, const int *seq_lens, int B,
+                            int Hq, int Hkv, int Nq, int max_pages, int page_size, int num_pages,
+                            int D, float scale, int causal, fav_dtype dtype, void *stream) {
+    if (!q || !k_cache || !v_cache || !o || !block_table || !seq_lens) return FAV_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(o, 16))
+        return FAV_ERR_INVALID_ARG;
+    if ((lse && !aligned(lse, 4)) || !aligned(block_table, 4) || !aligned(seq_lens, 4))
+        return FAV_ERR_INVALID_ARG;
+    if (max_pages <= 0 || num_pages <= 0 || page_size <= 0) return FAV_ERR_INVALID_ARG;
+    // pages of 16 .. 65536 rows, a power of two: a key tile then lies in one page, or a page
+    // holds whole 1024-byte swizzle atoms of a tile
+    if (page_size < 16 || page_size > 65536 || (page_size & (page_size - 1)) != 0)
+        return FAV_ERR_UNSUPPORTED;
+    const long long max_len = (long long)max_pages * page_size;
+    if (max_len > 0x7fffffffLL / 2) return FAV_ERR_UNSUPPORTED;
+    fav_status st = validate_shape(B, Hq, Hkv, Nq, (int)max_len, D, scale, causal, dtype);
+    if (st != FAV_OK) return st;
+    FavArgs a = make_args(q, k_cache, v_cache, o, lse, B, Hq, Hkv, Nq, (int)max_len, D, scale,
+                          causal, dtype);
+    if (!fav_decode_supported(a)) return FAV_ERR_UNSUPPORTED;
+    if ((long long)page_size * Hkv * D * 2 >= (1LL << 40)) return FAV_ERR_UNSUPPORTED;
+    DeviceState *ds = nullptr;
+    st = device_state(&ds);
+    if (st != FAV_OK) return st;
+    a.dev_status = ds->status;
+    a.num_sms = ds->num_sms;
+    const FavPaged pg{block_table, seq_lens, max_pages, page_size, num_pages};
+    // splits sized for the longest possible sequence; each block's boxes must fit its page list
+    const int tk = fav_decode_tile_keys(D);
+    const int n_tiles = fav_decode_num_tiles(a);
+    const int bpt = page_size >= tk ? 1 : tk / page_size;
+    int splits = g_splits.load();
+    if (splits <= 0) splits = fav_decode_auto_splits(a);
+    const long long min_splits =
+        ((long long)n_tiles * bpt + fav_decode_page_slots() - 1) / fav_decode_page_slots();
+    splits = (int)std::max<long long>(splits, min_splits);
+    splits = std::max(1, std::min(splits, n_tiles));
+    const int tps = (n_tiles + splits - 1) / splits;
+    splits = (n_tiles + tps - 1) / tps;
+    if ((long long)tps * bpt > fav_decode_page_slots()) return FAV_ERR_UNSUPPORTED;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaGetLastError();
+    void *ws = nullptr;
+    const size_t need = fav_decode_workspace_bytes(a, splits);
+    if (need) {
+        std::lock_guard<std::mutex> lk(g_mu);
+        st = ensure_buffer(&ds->ws, &ds->ws_bytes, need, s);
+        ws = ds->ws;
+    }
+    if (st == FAV_OK) st = fav_launch_decode_paged(a, pg, splits, ws, s);
+    if (st == FAV_OK) {
+        g_last_splits.store(splits);
+        g_last_path.store(FAV_PATH_DECODE);
+    }
+    return st;
+}
+
 fav_status fav_forward_strided(const void *q, const void *k, const void *v, void *o, float *lse,
                                fav_strides q_strides, fav_strides k_strides,
                                fav_strides v_strides, fav_strides o_strides, int B, int Hq,

@@ -27,7 +27,7 @@
 namespace {
 
 constexpr int kConsumers = 6;     // consumer warps
-constexpr int kThreads = (kConsumers + 1) * 32;
+constexpr int kThreads = (kConsumers + 2) * 32;   // + the K producer and the V producer
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -46,6 +46,9 @@ template <int D> struct DecodeCfg {
     static constexpr int kStageBytes = 2 * kTileBytes;
     static constexpr int kRingBytes = kStages * kStageBytes;
     static constexpr int kSmemBytes = kRingBytes + 1024 /*align*/ + 2 * kStages * 8;
+    // paged cache: the page id of every box this block loads, gathered once at the start
+    static constexpr int kPageSlots = 4096;
+    static constexpr int kSmemBytesPaged = kSmemBytes + 4 * kPageSlots;
     static_assert(kStages % kConsumers == 0, "stages must be owned by single warps");
     static_assert(kRingBytes >= kConsumers * 16 * D * 4 + 2 * kConsumers * 16 * 4,
                   "reduction buffer must fit in the ring");
@@ -58,14 +61,17 @@ __device__ __forceinline__ uint32_t swz(int j, int c) {
     return (uint32_t)((c >> 3) * (TK * 128) + j * 128 + (((c & 7) ^ (j & 7)) << 4));
 }
 
-template <typename T, int D>
+// kPaged: K and V are page pools ([num_pages, page_size, Hkv, D], tmK / tmV boxes of box_rows
+// rows); sequence b has min(seq_lens[b], max_pages * page_size) keys, and the producer warp
+// first gathers the page id of every box of the block's key range into shared memory.
+template <typename T, int D, bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
 fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                   const T *__restrict__ q, FavStrides qs, T *__restrict__ o, FavStrides os,
                   float *__restrict__ lse,
                   float *__restrict__ part_o, float *__restrict__ part_lse, int Hq, int Hkv,
                   int Nq, int Nkv, int n_tiles, int tiles_per_split, int splits,
-                  float scale_log2, int causal, int *status) {
+                  float scale_log2, int causal, int *status, FavPaged pg, int box_rows) {
     using Cfg = DecodeCfg<D>;
     constexpr int S = Cfg::kStages;
     constexpr int TK = Cfg::TK;
@@ -84,17 +90,25 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     const int G = Hq / Hkv;
     const int M = Nq * G;                        // query rows that read this KV head
     const int m0 = blockIdx.z * 16;
+    if constexpr (kPaged) {
+        // this sequence's length (clamped to its block-table row); tiles beyond it are empty
+        Nkv = min(max(pg.seq_lens[b], 0), pg.max_pages * pg.page_size);
+        n_tiles = (Nkv + TK - 1) / TK;
+    }
     const int tile0 = split * tiles_per_split;
-    const int my_tiles = min(tiles_per_split, n_tiles - tile0);
+    const int my_tiles = max(0, min(tiles_per_split, n_tiles - tile0));
+    int *page_list = reinterpret_cast<int *>(ring + Cfg::kRingBytes + 16 * S);
+    const int bpt = kPaged ? TK / box_rows : 1;               // boxes per tile and 64-column block
 
     // Let a dependent combine grid be scheduled once every block of this grid has started; it
     // still waits for this grid's completion before reading anything.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (threadIdx.x == 0) {
         (void)FAV_CHECK((ring_u32 & 1023u) == 0, status);
-        (void)FAV_CHECK((ring_u32 - raw_u32) + Cfg::kRingBytes + 16 * S <= fav::dynamic_smem_bytes(), status);
+        (void)FAV_CHECK((ring_u32 - raw_u32) + Cfg::kRingBytes + 16 * S +
+                            (kPaged ? 4 * Cfg::kPageSlots : 0) <= fav::dynamic_smem_bytes(), status);
         for (int s = 0; s < S; ++s) {
-            fav::mbar_init(full0 + 8 * s, 1);
+            fav::mbar_init(full0 + 8 * s, 2);          // the K and the V producer
             fav::mbar_init(empty0 + 8 * s, 1);
         }
         fav::mbar_fence_init();
@@ -110,28 +124,63 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
 #else
 #define FAV_DSTAMP(arr, lt) do { } while (0)
 #endif
-    if (warp == kConsumers) {
-        // ---------------- producer: one lane streams K/V tiles with TMA ----------------
+    if (warp >= kConsumers) {
+        // ---------------- producers: lane 0 of warp kConsumers streams K, of the next warp V
+        // (two issuing threads double the copy instructions a block can issue per unit time) --
+        const bool is_v = warp == kConsumers + 1;
+        const CUtensorMap *tm = is_v ? &tmV : &tmK;
+        if constexpr (kPaged) {
+            // page id of box e (tile e / bpt, rows (e % bpt) * box_rows .. + box_rows); boxes
+            // past the sequence read page 0 (their keys are masked).  Filled by the K warp;
+            // both producer warps then meet at a named barrier (neither leaves before it).
+            if (!is_v) {
+                const int n_box = my_tiles * bpt;
+                for (int e = lane; e < n_box && e < Cfg::kPageSlots; e += 32) {
+                    const int key = (tile0 + e / bpt) * TK + (e % bpt) * box_rows;
+                    page_list[e] = key < Nkv ? pg.block_table[(long long)b * pg.max_pages + key / pg.page_size] : 0;
+                }
+            }
+            fav::named_bar_sync(2, 64);
+        }
         if (lane == 0) {
-            fav::tma_prefetch_desc(&tmK);
-            fav::tma_prefetch_desc(&tmV);
+            fav::tma_prefetch_desc(tm);
             for (int lt = 0; lt < my_tiles; ++lt) {
                 const int st = lt % S;
                 if (lt >= S && !fav::mbar_wait(empty0 + 8 * st, ((lt / S) - 1) & 1, status)) break;
                 const uint32_t full = full0 + 8 * st;
-                FAV_DSTAMP(t_issue, lt);
-                fav::mbar_arrive_expect_tx(full, Cfg::kStageBytes);
+                if (!is_v) FAV_DSTAMP(t_issue, lt);
+                fav::mbar_arrive_expect_tx(full, Cfg::kTileBytes);
                 const int key0 = (tile0 + lt) * TK;
-                const uint32_t kdst = ring_u32 + st * Cfg::kStageBytes;
-                const uint32_t vdst = kdst + Cfg::kTileBytes;
+                const uint32_t dst = ring_u32 + st * Cfg::kStageBytes + (is_v ? Cfg::kTileBytes : 0);
+                if (!FAV_CHECK(dst + Cfg::kBoxes * TK * 128 <= ring_u32 + Cfg::kRingBytes &&
+                                   (dst & 1023u) == 0 && key0 < n_tiles * TK &&
+                                   bkv < (int)gridDim.y, status))
+                    continue;
+                // One copy instruction per box: the tensor maps are 5-D views whose box covers
+                // all D / 64 column blocks (each TK x 128 bytes in shared memory; a copy
+                // instruction costs the producer the same time whatever its size).
+                if constexpr (kPaged) {
+                    // bpt boxes of box_rows rows, each inside one page (row offsets keep the
+                    // 1024-byte swizzle atoms aligned: box_rows >= 16); page sizes are powers
+                    // of two, so the row in the page is a mask.  A box shorter than the tile
+                    // (bpt > 1) with several column blocks is copied block by block (4-D maps):
+                    // a 5-D box would pack its blocks box_rows (not TK) rows apart.
+                    for (int i = 0; i < bpt; ++i) {
+                        const int e = lt * bpt + i;
+                        if (!FAV_CHECK(e < Cfg::kPageSlots, status)) continue;
+                        const int pid = page_list[e];
+                        const int row = (key0 + i * box_rows) & (pg.page_size - 1);
+                        if (Cfg::kBoxes == 1 || bpt == 1) {
+                            fav::tma_load_5d(dst + i * box_rows * 128, tm, full, 0, row, 0, g, pid);
+                        } else {
 #pragma unroll
-                for (int bx = 0; bx < Cfg::kBoxes; ++bx) {
-                    if (!FAV_CHECK(vdst + (bx + 1) * TK * 128 <= ring_u32 + Cfg::kRingBytes &&
-                                       ((kdst | vdst) & 1023u) == 0 && key0 < n_tiles * TK &&
-                                       bkv < (int)gridDim.y, status))
-                        continue;
-                    fav::tma_load_4d(kdst + bx * TK * 128, &tmK, full, bx * 64, key0, g, b);
-                    fav::tma_load_4d(vdst + bx * TK * 128, &tmV, full, bx * 64, key0, g, b);
+                            for (int bx = 0; bx < Cfg::kBoxes; ++bx)
+                                fav::tma_load_4d(dst + bx * TK * 128 + i * box_rows * 128, tm, full,
+                                                 bx * 64, row, g, pid);
+                        }
+                    }
+                } else {
+                    fav::tma_load_5d(dst, tm, full, 0, key0, 0, g, b);
                 }
             }
         }
@@ -423,26 +472,24 @@ fav_combine_kernel(const float *__restrict__ part_o, const float *__restrict__ p
     if (lse && threadIdx.x == 0) lse[row] = L;
 }
 
-template <typename T, int D>
-fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t stream) {
+// Shared by the dense and paged launches: the decode grid (splits, B * Hkv, 16-row chunks)
+// and, with several splits, the combine kernel as a programmatic dependent launch.
+template <typename T, int D, bool kPaged>
+fav_status launch_grids(const FavArgs &a, const CUtensorMap &tmK, const CUtensorMap &tmV,
+                        int n_tiles, int splits, void *workspace, cudaStream_t stream,
+                        const FavPaged &pg, int box_rows) {
     using Cfg = DecodeCfg<D>;
-    constexpr int TK = Cfg::TK;
-    alignas(64) CUtensorMap tmK, tmV;
-    const int outer = a.B * a.Hkv;
-    fav_status st = fav_make_tmap_4d(&tmK, a.k, D, a.Nkv, a.Hkv, a.B, a.ks, TK);
-    if (st != FAV_OK) return st;
-    st = fav_make_tmap_4d(&tmV, a.v, D, a.Nkv, a.Hkv, a.B, a.vs, TK);
-    if (st != FAV_OK) return st;
-    const int n_tiles = fav_decode_num_tiles(a);
     const int tps = (n_tiles + splits - 1) / splits;
     splits = (n_tiles + tps - 1) / tps;
+    const int outer = a.B * a.Hkv;
     const int M = a.Nq * (a.Hq / a.Hkv);
     const int chunks = (M + 15) / 16;
-    auto kern = fav_decode_kernel<T, D>;
+    auto kern = fav_decode_kernel<T, D, kPaged>;
+    constexpr int smem = kPaged ? Cfg::kSmemBytesPaged : Cfg::kSmemBytes;
     static bool attr_set = false;   // per-process; the attribute is per function, not per device
     if (!attr_set) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 Cfg::kSmemBytes) != cudaSuccess)
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+            cudaSuccess)
             return FAV_ERR_CUDA;
         attr_set = true;
     }
@@ -451,9 +498,9 @@ fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t st
     float *part_lse = part_o ? part_o + rows * splits * D : nullptr;
     const float scale_log2 = a.scale * kLog2e;
     dim3 grid(splits, outer, chunks);
-    kern<<<grid, kThreads, Cfg::kSmemBytes, stream>>>(
-        tmK, tmV, (const T *)a.q, a.qs, (T *)a.o, a.os, a.lse, part_o, part_lse, a.Hq, a.Hkv, a.Nq, a.Nkv,
-        n_tiles, tps, splits, scale_log2, a.causal, a.dev_status);
+    kern<<<grid, kThreads, smem, stream>>>(
+        tmK, tmV, (const T *)a.q, a.qs, (T *)a.o, a.os, a.lse, part_o, part_lse, a.Hq, a.Hkv,
+        a.Nq, a.Nkv, n_tiles, tps, splits, scale_log2, a.causal, a.dev_status, pg, box_rows);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_decode_kernel", stream))
         return FAV_ERR_CUDA;
     if (splits > 1) {
@@ -476,6 +523,43 @@ fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t st
             return FAV_ERR_CUDA;
     }
     return FAV_OK;
+}
+
+template <typename T, int D>
+fav_status launch(const FavArgs &a, int splits, void *workspace, cudaStream_t stream) {
+    constexpr int TK = DecodeCfg<D>::TK;
+    alignas(64) CUtensorMap tmK, tmV;
+    fav_status st = fav_make_tmap_tiles(&tmK, a.k, D, a.Nkv, a.Hkv, a.B, a.ks, TK);
+    if (st != FAV_OK) return st;
+    st = fav_make_tmap_tiles(&tmV, a.v, D, a.Nkv, a.Hkv, a.B, a.vs, TK);
+    if (st != FAV_OK) return st;
+    const FavPaged none{nullptr, nullptr, 0, 0, 0};
+    return launch_grids<T, D, false>(a, tmK, tmV, fav_decode_num_tiles(a), splits, workspace,
+                                     stream, none, TK);
+}
+
+// Paged cache: the pools viewed as [num_pages][page_size][Hkv][D] -- a 4-D tensor (D,
+// page_size, Hkv, num_pages) with boxes of min(page_size, TK) rows of one head of one page.
+template <typename T, int D>
+fav_status launch_paged(const FavArgs &a, const FavPaged &pg, int splits, void *workspace,
+                        cudaStream_t stream) {
+    constexpr int TK = DecodeCfg<D>::TK;
+    const int box_rows = std::min(pg.page_size, TK);
+    const FavStrides ps{(long long)pg.page_size * a.Hkv * D, (long long)D, (long long)a.Hkv * D};
+    alignas(64) CUtensorMap tmK, tmV;
+    // one 5-D box per page piece when it spans the whole tile or D has one column block; 4-D
+    // per-block boxes otherwise (the kernel makes the same choice)
+    const bool tiles5 = (D == 64) || (box_rows == TK);
+    auto make = [&](CUtensorMap *m, const void *base) {
+        return tiles5 ? fav_make_tmap_tiles(m, base, D, pg.page_size, a.Hkv, pg.num_pages, ps, box_rows)
+                      : fav_make_tmap_4d(m, base, D, pg.page_size, a.Hkv, pg.num_pages, ps, box_rows);
+    };
+    fav_status st = make(&tmK, a.k);
+    if (st != FAV_OK) return st;
+    st = make(&tmV, a.v);
+    if (st != FAV_OK) return st;
+    return launch_grids<T, D, true>(a, tmK, tmV, fav_decode_num_tiles(a), splits, workspace,
+                                    stream, pg, box_rows);
 }
 
 }  // namespace
@@ -513,6 +597,18 @@ size_t fav_decode_workspace_bytes(const FavArgs &a, int splits) {
     if (splits <= 1) return 0;
     const size_t rows = (size_t)a.B * a.Hq * a.Nq;
     return rows * splits * ((size_t)a.D + 1) * sizeof(float);
+}
+
+int fav_decode_tile_keys(int D) { return D == 128 ? DecodeCfg<128>::TK : DecodeCfg<64>::TK; }
+int fav_decode_page_slots() { return DecodeCfg<128>::kPageSlots; }
+
+fav_status fav_launch_decode_paged(const FavArgs &a, const FavPaged &pg, int splits,
+                                   void *workspace, cudaStream_t s) {
+    if (a.dtype == FAV_F16)
+        return a.D == 128 ? launch_paged<__half, 128>(a, pg, splits, workspace, s)
+                          : launch_paged<__half, 64>(a, pg, splits, workspace, s);
+    return a.D == 128 ? launch_paged<__nv_bfloat16, 128>(a, pg, splits, workspace, s)
+                      : launch_paged<__nv_bfloat16, 64>(a, pg, splits, workspace, s);
 }
 
 fav_status fav_launch_decode(const FavArgs &a, int splits, void *workspace, cudaStream_t s) {

@@ -34,6 +34,20 @@ int fav_decode_num_tiles(const FavArgs &a);
 int fav_decode_auto_splits(const FavArgs &a);
 size_t fav_decode_workspace_bytes(const FavArgs &a, int splits);
 fav_status fav_launch_decode(const FavArgs &a, int splits, void *workspace, cudaStream_t s);
+// Paged KV cache for the decode kernel: K and V are pools of num_pages pages of
+// [page_size, Hkv, D]; sequence b's key n lives in page block_table[b * max_pages +
+// n / page_size], row n % page_size; sequence b has seq_lens[b] keys (device arrays).
+struct FavPaged {
+    const int *block_table;
+    const int *seq_lens;
+    int max_pages, page_size, num_pages;
+};
+// Keys per tile of the decode kernel at head dimension D, and the capacity (page references
+// per thread block) of its page list: a split must cover at most that many boxes.
+int fav_decode_tile_keys(int D);
+int fav_decode_page_slots();
+fav_status fav_launch_decode_paged(const FavArgs &a, const FavPaged &pg, int splits,
+                                   void *workspace, cudaStream_t s);
 
 // tcgen05 prefill kernel (fav_prefill.cu).
 bool fav_prefill_supported(const FavArgs &a);
