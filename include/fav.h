@@ -118,6 +118,29 @@ FAV_API fav_status fav_forward_strided(const void *q, const void *k, const void 
                                        int causal, fav_dtype dtype, void *stream);
 
 /*
+ * fav_prefill_varlen -- prefill attention over a batch of sequences of different lengths packed
+ * one after another (the cu_seqlens layout), in one launch of the persistent prefill kernel.
+ * (Method / experiments: prompts of different lengths; each sequence attends only to itself.)
+ *
+ *  q, o           device, [total_q, Hq, D] contiguous (token-major, the heads of a token side by
+ *                 side), `dtype`, 16-byte aligned; total_q = cu_seqlens_q[B]
+ *  k, v           device, [total_k, Hkv, D] contiguous, `dtype`, 16-byte aligned
+ *  lse            device [Hq, total_q] fp32, or NULL
+ *  cu_seqlens_q,  HOST int32 [B + 1], non-decreasing from 0: sequence b's queries are rows
+ *  cu_seqlens_k   cu_seqlens_q[b] .. cu_seqlens_q[b+1]-1 of q (keys likewise of k and v).  A
+ *                 sequence with queries needs at least one key; causal (bottom-right aligned per
+ *                 sequence) needs no more queries than keys; else FAV_ERR_INVALID_ARG.
+ *  dtype, D       fp16 or bf16 with D = 128 (else FAV_ERR_UNSUPPORTED)
+ *  other arguments as fav_forward.  The library builds the kernel's work list from the host
+ *  arrays and copies it to a device buffer on `stream` (returning once the copy is staged);
+ *  the call is otherwise asynchronous on `stream`.  total_q = 0 computes nothing.
+ */
+FAV_API fav_status fav_prefill_varlen(const void *q, const void *k, const void *v, void *o,
+                                      float *lse, const int *cu_seqlens_q,
+                                      const int *cu_seqlens_k, int B, int Hq, int Hkv, int D,
+                                      float scale, int causal, fav_dtype dtype, void *stream);
+
+/*
  * fav_decode_paged -- decode (and small-Nq) attention over a PAGED key/value cache, per sequence
  * of its own length.  (Method section: the decode stage attends one query row per head to the
  * whole cached sequence; a serving system keeps that cache in fixed-size pages shared by many

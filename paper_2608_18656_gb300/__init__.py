@@ -7,7 +7,7 @@ CPU fallback: without the built library every call raises.
 import ctypes
 import os
 
-__all__ = ["forward", "forward_host", "decode_paged", "Strides", "set_path", "last_path", "set_decode_splits",
+__all__ = ["forward", "forward_host", "decode_paged", "prefill_varlen", "Strides", "set_path", "last_path", "set_decode_splits",
            "last_decode_splits", "set_prefill_grid", "device_status", "release_workspace", "library_path",
            "FavError", "F32", "F16", "BF16", "PATH_AUTO", "PATH_SIMT", "PATH_DECODE",
            "PATH_PREFILL"]
@@ -60,6 +60,9 @@ def lib():
         L.fav_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i, i, i,
                                        ctypes.c_float, i, i, vp]
         L.fav_decode_paged.restype = i
+        L.fav_prefill_varlen.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, ctypes.c_float,
+                                         i, i, vp]
+        L.fav_prefill_varlen.restype = i
         L.fav_status_string.argtypes = [i]
         L.fav_status_string.restype = ctypes.c_char_p
         L.fav_get_last_device_status.argtypes = []
@@ -182,6 +185,47 @@ def decode_paged(q, k_cache, v_cache, block_table, seq_lens, causal=False, scale
                                     block_table.data_ptr(), seq_lens.data_ptr(), B, Hq, Hkv, Nq,
                                     max_pages, page_size, num_pages, D, float(scale),
                                     int(bool(causal)), _dtype_code(q), s.cuda_stream)
+    _check(st)
+    return o, lse
+
+
+def prefill_varlen(q, k, v, cu_seqlens_q, cu_seqlens_k, causal=False, scale=None,
+                   return_lse=True, out=None, lse_out=None, stream=None):
+    """Prefill over a packed batch of variable-length sequences (fav_prefill_varlen).
+
+    q [total_q, Hq, D], k / v [total_k, Hkv, D]: contiguous torch CUDA tensors; cu_seqlens_q /
+    cu_seqlens_k: length-B+1 host sequences of ints (lists, numpy arrays or CPU tensors).
+    Returns (o [total_q, Hq, D], lse [Hq, total_q] fp32 or None).
+    """
+    import numpy as np
+    import torch
+    for t in (q, k, v):
+        if not t.is_cuda or not t.is_contiguous() or t.dim() != 3:
+            raise ValueError("q, k, v must be contiguous 3-D CUDA tensors")
+    if k.dtype != q.dtype or v.dtype != q.dtype:
+        raise TypeError("q, k and v must share a dtype")
+    cq = np.ascontiguousarray(np.asarray(cu_seqlens_q, dtype=np.int32))
+    ck = np.ascontiguousarray(np.asarray(cu_seqlens_k, dtype=np.int32))
+    if cq.ndim != 1 or cq.shape != ck.shape or cq.size < 2:
+        raise ValueError("cu_seqlens_q and cu_seqlens_k must both have B + 1 entries")
+    B = cq.size - 1
+    total_q, Hq, D = q.shape
+    total_k, Hkv, Dk = k.shape
+    if tuple(v.shape) != tuple(k.shape) or Dk != D or cq[-1] != total_q or ck[-1] != total_k:
+        raise ValueError("shape mismatch between q, k, v and the sequence offsets")
+    if scale is None:
+        scale = float(np.float32(1.0 / np.sqrt(D)))
+    o = out if out is not None else torch.empty(q.shape, dtype=q.dtype, device=q.device)
+    lse = None
+    if return_lse:
+        lse = lse_out if lse_out is not None else torch.empty((Hq, total_q), device=q.device,
+                                                              dtype=torch.float32)
+    s = stream if stream is not None else torch.cuda.current_stream(q.device)
+    with torch.cuda.device(q.device):
+        st = lib().fav_prefill_varlen(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(),
+                                      lse.data_ptr() if lse is not None else None,
+                                      cq.ctypes.data, ck.ctypes.data, B, Hq, Hkv, D, float(scale),
+                                      int(bool(causal)), _dtype_code(q), s.cuda_stream)
     _check(st)
     return o, lse
 

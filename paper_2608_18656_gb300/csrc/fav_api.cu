@@ -9,6 +9,7 @@
 #include <stdlib.h>
 
 #include <algorithm>
+#include <vector>
 #include <atomic>
 #include <mutex>
 
@@ -29,6 +30,8 @@ struct DeviceState {
     size_t ws_bytes = 0;
     void *ws_pre = nullptr;    // prefill workspace (bf16: fp16 copy of V and its scales)
     size_t ws_pre_bytes = 0;
+    void *ws_units = nullptr;  // unit table of a packed variable-length prefill
+    size_t ws_units_bytes = 0;
     void *hbuf = nullptr;      // device copies for fav_forward_host
     size_t hbuf_bytes = 0;
     bool pipe_init = false;    // fav_forward_host pipeline: copy-in, compute, copy-out streams
@@ -291,6 +294,88 @@ fav_status fav_forward(const void *q, const void *k, const void *v, void *o, flo
     return forward_impl(a, static_cast<cudaStream_t>(stream));
 }
 
+fav_status fav_prefill_varlen(const void *q, const void *k, const void *v, void *o, float *lse,
+                              const int *cu_seqlens_q, const int *cu_seqlens_k, int B, int Hq,
+                              int Hkv, int D, float scale, int causal, fav_dtype dtype,
+                              void *stream) {
+    if (!q || !k || !v || !o || !cu_seqlens_q || !cu_seqlens_k) return FAV_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(o, 16))
+        return FAV_ERR_INVALID_ARG;
+    if (lse && !aligned(lse, 4)) return FAV_ERR_INVALID_ARG;
+    if (B <= 0 || (causal != 0 && causal != 1)) return FAV_ERR_INVALID_ARG;
+    if (cu_seqlens_q[0] != 0 || cu_seqlens_k[0] != 0) return FAV_ERR_INVALID_ARG;
+    for (int b = 0; b < B; ++b) {
+        const int lq = cu_seqlens_q[b + 1] - cu_seqlens_q[b];
+        const int lk = cu_seqlens_k[b + 1] - cu_seqlens_k[b];
+        if (cu_seqlens_q[b + 1] < cu_seqlens_q[b] || cu_seqlens_k[b + 1] < cu_seqlens_k[b])
+            return FAV_ERR_INVALID_ARG;
+        if (lq > 0 && lk == 0) return FAV_ERR_INVALID_ARG;   // queries with no key at all
+        if (causal && lq > lk) return FAV_ERR_INVALID_ARG;   // bottom-right alignment
+    }
+    const int total_q = cu_seqlens_q[B], total_k = cu_seqlens_k[B];
+    fav_status st = validate_shape(1, Hq, Hkv, std::max(total_q, 1), std::max(total_k, 1), D,
+                                   scale, 0, dtype);
+    if (st != FAV_OK) return st;
+    if ((dtype != FAV_F16 && dtype != FAV_BF16) || D != 128) return FAV_ERR_UNSUPPORTED;
+    if (total_q == 0) return FAV_OK;                       // nothing to compute
+    // units: one 128-row query tile of one head of one sequence, heaviest causal work first
+    // (then sequence, tile, head: the heads of a GQA group side by side), as in the dense kernel
+    struct U { int s, h, t, n_kv, q0, k0, lq, lk; };
+    std::vector<U> units;
+    for (int b = 0; b < B; ++b) {
+        const int lq = cu_seqlens_q[b + 1] - cu_seqlens_q[b];
+        const int lk = cu_seqlens_k[b + 1] - cu_seqlens_k[b];
+        for (int t = 0; t * 128 < lq; ++t) {
+            const int kv_end = causal ? std::min(lk, t * 128 + 128 + lk - lq) : lk;
+            const int n_kv = (kv_end + 127) / 128;
+            for (int h = 0; h < Hq; ++h)
+                units.push_back(U{b, h, t, n_kv, cu_seqlens_q[b], cu_seqlens_k[b], lq, lk});
+        }
+    }
+    if (units.size() + 4096 > 0x7fffffffu) return FAV_ERR_UNSUPPORTED;
+    std::stable_sort(units.begin(), units.end(), [](const U &x, const U &y) {
+        if (x.n_kv != y.n_kv) return x.n_kv > y.n_kv;
+        if (x.s != y.s) return x.s < y.s;
+        if (x.t != y.t) return x.t < y.t;
+        return x.h < y.h;
+    });
+    std::vector<int> table(units.size() * 8);
+    for (size_t i = 0; i < units.size(); ++i) {
+        const U &u = units[i];
+        const int e[8] = {u.s, u.h, u.t, u.n_kv, u.q0, u.k0, u.lq, u.lk};
+        std::copy(e, e + 8, table.begin() + 8 * i);
+    }
+    FavArgs a = make_args(q, k, v, o, lse, 1, Hq, Hkv, total_q, total_k, D, scale, causal, dtype);
+    a.qs = a.os = FavStrides{(long long)total_q * Hq * D, (long long)D, (long long)Hq * D};
+    a.ks = a.vs = FavStrides{(long long)total_k * Hkv * D, (long long)D, (long long)Hkv * D};
+    DeviceState *ds = nullptr;
+    st = device_state(&ds);
+    if (st != FAV_OK) return st;
+    a.dev_status = ds->status;
+    a.num_sms = ds->num_sms;
+    a.prefill_grid = g_prefill_grid.load();
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaGetLastError();
+    void *ws = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        const size_t tb = table.size() * sizeof(int);
+        st = ensure_buffer(&ds->ws_units, &ds->ws_units_bytes, tb, s);
+        // (pageable source: the call returns once the table has been staged for the copy)
+        if (st == FAV_OK && cudaMemcpyAsync(ds->ws_units, table.data(), tb,
+                                            cudaMemcpyHostToDevice, s) != cudaSuccess)
+            st = FAV_ERR_CUDA;
+        const size_t need = fav_prefill_workspace_bytes(a);
+        if (st == FAV_OK && need) st = ensure_buffer(&ds->ws_pre, &ds->ws_pre_bytes, need, s);
+        ws = ds->ws_pre;
+    }
+    if (st == FAV_OK)
+        st = fav_launch_prefill_varlen(a, static_cast<const int4 *>(ds->ws_units),
+                                       (int)units.size(), ws, s);
+    if (st == FAV_OK) g_last_path.store(FAV_PATH_PREFILL);
+    return st;
+}
+
 fav_status fav_decode_paged(const void *q, const void *k_cache, const void *v_cache, void *o,
                             float *lse, const int *block_table, const int *seq_lens, int B,
                             int Hq, int Hkv, int Nq, int max_pages, int page_size, int num_pages,
@@ -502,8 +587,9 @@ void fav_release_workspace(void) {
     if (d.ws) cudaFree(d.ws);
     if (d.ws_pre) cudaFree(d.ws_pre);
     if (d.hbuf) cudaFree(d.hbuf);
-    d.ws = d.ws_pre = d.hbuf = nullptr;
-    d.ws_bytes = d.ws_pre_bytes = d.hbuf_bytes = 0;
+    if (d.ws_units) cudaFree(d.ws_units);
+    d.ws = d.ws_pre = d.hbuf = d.ws_units = nullptr;
+    d.ws_bytes = d.ws_pre_bytes = d.hbuf_bytes = d.ws_units_bytes = 0;
 }
 
 fav_status fav_set_path(fav_path p) {

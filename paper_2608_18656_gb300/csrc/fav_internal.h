@@ -63,6 +63,12 @@ fav_status fav_v16_convert(const FavArgs &a, void *workspace, cudaStream_t strea
 // The two prefill kernel designs (fav_prefill.cu: D = 128; fav_prefill_pair.cu: D = 64).
 fav_status fav_launch_prefill_split(const FavArgs &a, void *workspace, cudaStream_t s);
 fav_status fav_launch_prefill_pair(const FavArgs &a, void *workspace, cudaStream_t s);
+// Packed variable-length batch (D = 128): a is the [1, H, total, D] view of the packed tensors
+// (Nq = total_q, Nkv = total_k, token strides H * D); units is the device table built by
+// fav_prefill_varlen, two int4 per unit: {sequence, head, query tile, key tiles},
+// {first query row, first key row, query length, key length}, heaviest causal work first.
+fav_status fav_launch_prefill_varlen(const FavArgs &a, const int4 *units, int n_units,
+                                     void *workspace, cudaStream_t s);
 fav_status fav_launch_prefill(const FavArgs &a, void *workspace, cudaStream_t s);
 
 // With FAV_DEBUG_SYNC=1 in the environment: synchronise `s` after a launch and report a

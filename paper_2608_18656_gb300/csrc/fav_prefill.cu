@@ -127,8 +127,8 @@ template <int D> struct PrefillCfg {
     static constexpr int kOffV = kOffK + kKStages * kKVBytes;
     static constexpr int kOffXch = kOffV + kVStages * kKVBytes;   // (m, l) [2][4][splits][32]
     static constexpr int kXchBytes = 2 * 4 * kSplits * 32 * 8;
-    static constexpr int kOffUnits = kOffXch + kXchBytes;         // int[kUnitTab][8]
-    static constexpr int kOffBar = kOffUnits + kUnitTab * 32;
+    static constexpr int kOffUnits = kOffXch + kXchBytes;         // int[kUnitTab][12]
+    static constexpr int kOffBar = kOffUnits + kUnitTab * 48;
     static constexpr int kNumBars = 2 + 2 + 2 * kKStages + 2 * kVStages + 2 + 2 + 2 + 2 + 2 + 1;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
     static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
@@ -147,9 +147,11 @@ __global__ void __launch_bounds__(PrefillCfg<D>::kThreads, 1)
 fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                          const __grid_constant__ CUtensorMap tmK,
                          const __grid_constant__ CUtensorMap tmV,
-                         const __grid_constant__ CUtensorMap tmO, float *__restrict__ lse, const float *__restrict__ v_scale, int B, int Hq,
-                   int Hkv, int Nq, int Nkv, int n_qtiles, float scale_log2, int causal,
-                   int *status) {
+                         const __grid_constant__ CUtensorMap tmO, T *__restrict__ o,
+                         FavStrides os, float *__restrict__ lse,
+                         const float *__restrict__ v_scale, int B, int Hq, int Hkv, int Nq,
+                         int Nkv, int n_qtiles, float scale_log2, int causal, int *status,
+                         const int4 *__restrict__ vunits, int n_vunits) {
     using C = PrefillCfg<D>;
     using TP = __half;    // type of the weights P and of V in shared memory (P.V MMA)
     constexpr int KS = C::kKStages, VS = C::kVStages, NS = C::kSplits, SK = C::kSplitKeys;
@@ -184,10 +186,16 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     // Unit u: query tile t = n_qtiles - 1 - u / (B * Hq) of head (b, h) = u % (B * Hq), so the
     // heads of one GQA group (consecutive h) run side by side.  The CTA takes units c, 2P-1-c,
     // 2P+c, 4P-1-c, ... (P CTAs, "snake" order), which evens out the work per CTA.
+    // Variable-length batches (vunits != null): the units come from a table built on the host
+    // (sorted the same way), Q/O are [1, Hq, total_q, D] and K/V [1, Hkv, total_k, D] views of
+    // the packed tensors, and a unit's rows start at its sequence's offsets q_y0 / k_y0.
+    // Unit: TMA batch coordinate b, head h, query tile t of its sequence, key tiles n_kv, KV head
+    // kvh, sequence offsets and lengths.
     struct Unit {
-        int b, h, t, n_kv, kvh;
+        int b, h, t, n_kv, kvh, q_y0, k_y0, len_q, len_k;
     };
-    const int n_units = n_qtiles * BH;
+    const bool varlen = vunits != nullptr;
+    const int n_units = varlen ? n_vunits : n_qtiles * BH;
     auto unit_at = [&](int k) {   // the k-th unit of this CTA, or -1
         const int P = gridDim.x, c = blockIdx.x;
         const int u = k * P + ((k & 1) ? (P - 1 - c) : c);
@@ -195,22 +203,38 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     };
     auto make_unit = [&](int u) {
         Unit U;
-        const int bh = u % BH;
-        U.t = n_qtiles - 1 - u / BH;
-        U.b = bh / Hq;
-        U.h = bh % Hq;
+        if (varlen) {
+            const int4 a = vunits[2 * u], c = vunits[2 * u + 1];
+            U.b = 0;
+            U.h = a.y;
+            U.t = a.z;
+            U.n_kv = a.w;
+            U.q_y0 = c.x;
+            U.k_y0 = c.y;
+            U.len_q = c.z;
+            U.len_k = c.w;
+        } else {
+            const int bh = u % BH;
+            U.t = n_qtiles - 1 - u / BH;
+            U.b = bh / Hq;
+            U.h = bh % Hq;
+            U.q_y0 = U.k_y0 = 0;
+            U.len_q = Nq;
+            U.len_k = Nkv;
+            const int kv_end = causal ? min(Nkv, U.t * BM + BM + off) : Nkv;
+            U.n_kv = (kv_end + BN - 1) / BN;
+        }
         U.kvh = U.h / G;
-        const int kv_end = causal ? min(Nkv, U.t * BM + BM + off) : Nkv;
-        U.n_kv = (kv_end + BN - 1) / BN;
         return U;
     };
     // The CTA's first kUnitTab units are computed once, in parallel, into shared memory (the
     // integer divisions would otherwise sit on the critical path at every unit switch).
     auto unit = [&](int k) {
         if (k < C::kUnitTab) {
-            const int *e = utab + 8 * k;
+            const int *e = utab + 12 * k;
             Unit U;
             U.b = e[0]; U.h = e[1]; U.t = e[2]; U.n_kv = e[3]; U.kvh = e[4];
+            U.q_y0 = e[5]; U.k_y0 = e[6]; U.len_q = e[7]; U.len_k = e[8];
             return U;
         }
         return make_unit(unit_at(k));
@@ -259,18 +283,19 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         fav::tma_prefetch_desc(&tmK);
         const Unit U0 = make_unit(unit_at(0));
         fav::mbar_arrive_expect_tx(q_full, C::kQBytes);
-        fav::tma_load_5d(sQ, &tmQ, q_full, 0, U0.t * BM, 0, U0.h, U0.b);
+        fav::tma_load_5d(sQ, &tmQ, q_full, 0, U0.q_y0 + U0.t * BM, 0, U0.h, U0.b);
         for (int g = 0; g < KS && g < U0.n_kv; ++g) {
             fav::mbar_arrive_expect_tx(k_full + 8 * g, C::kKVBytes);
-            fav::tma_load_5d(sK + g * C::kKVBytes, &tmK, k_full + 8 * g, 0, g * BN, 0, U0.kvh, U0.b);
+            fav::tma_load_5d(sK + g * C::kKVBytes, &tmK, k_full + 8 * g, 0, U0.k_y0 + g * BN, 0, U0.kvh, U0.b);
         }
     }
     for (int k = threadIdx.x; k < C::kUnitTab; k += blockDim.x) {
         const int u = unit_at(k);
         if (u < 0) break;
         const Unit U = make_unit(u);
-        int *e = utab + 8 * k;
+        int *e = utab + 12 * k;
         e[0] = U.b; e[1] = U.h; e[2] = U.t; e[3] = U.n_kv; e[4] = U.kvh;
+        e[5] = U.q_y0; e[6] = U.k_y0; e[7] = U.len_q; e[8] = U.len_k;
     }
 
 #ifdef FAV_TIMING
@@ -312,8 +337,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             const Unit U = unit(k);
             const int q0 = U.t * BM;
             const int qi = q0 + row;                          // query index of this row
-            const int lim = causal ? min(Nkv, qi + off + 1) : Nkv;       // visible keys: [0, lim)
-            const int lim_tile = causal ? min(Nkv, q0 + off + 1) : Nkv;  // smallest lim in the tile
+            const int uoff = U.len_k - U.len_q;               // bottom-right causal offset
+            const int lim = causal ? min(U.len_k, qi + uoff + 1) : U.len_k;      // visible keys: [0, lim)
+            const int lim_tile = causal ? min(U.len_k, q0 + uoff + 1) : U.len_k; // smallest lim in the tile
             float m = -INFINITY, l = 0.f;
             for (int j = 0; j < U.n_kv; ++j, ++Gt) {
                 FAV_TSS(0);
@@ -465,6 +491,11 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             const float inv_l = vsc / L;
             const float a0 = w0 * inv_l, a1 = w1 * inv_l;
             const uint32_t stage = sQ + (k & 1) * C::kQBytes + row * 128;
+            // the last tile of a packed sequence is written row by row (its rows past the end
+            // belong to the next sequence); every other tile goes through the TMA store
+            const bool partial = varlen && U.t * BM + BM > U.len_q;
+            const bool valid = qi < U.len_q;
+            T *orow = o + U.b * os.b + U.h * os.h + (long long)(U.q_y0 + qi) * os.n;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {   // 32 columns at a time, both splits in flight
                 uint32_t v0[32], v1[32];
@@ -483,11 +514,15 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                             fmaf(a0, __uint_as_float(v0[i]), a1 * __uint_as_float(v1[i])),
                             fmaf(a0, __uint_as_float(v0[i + 1]), a1 * __uint_as_float(v1[i + 1])));
                     }
-                    const uint32_t chunk = (uint32_t)(4 * (c & 1) + h) ^ (uint32_t)(row & 7);
-                    const uint32_t addr = stage + (c >> 1) * (BM * 128) + (chunk << 4);
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};"
-                                 ::"r"(addr), "r"(x[0]), "r"(x[1]), "r"(x[2]), "r"(x[3])
-                                 : "memory");
+                    if (!partial) {
+                        const uint32_t chunk = (uint32_t)(4 * (c & 1) + h) ^ (uint32_t)(row & 7);
+                        const uint32_t addr = stage + (c >> 1) * (BM * 128) + (chunk << 4);
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};"
+                                     ::"r"(addr), "r"(x[0]), "r"(x[1]), "r"(x[2]), "r"(x[3])
+                                     : "memory");
+                    } else if (valid) {
+                        *reinterpret_cast<uint4 *>(orow + c * 32 + 8 * h) = make_uint4(x[0], x[1], x[2], x[3]);
+                    }
                 }
             }
             // O has been read: release it to the next unit's first P.V
@@ -495,8 +530,12 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             fav::mbar_arrive(o_free);
             fav::tc::fence_proxy_async_smem();   // visible to the TMA store (async proxy)
             fav::mbar_arrive(o_staged + 8 * (k & 1));
-            if (qi < Nq && lse)
-                lse[(long long)(U.b * Hq + U.h) * Nq + qi] = (Mx - kPShift + log2f(L)) * kLn2;
+            if (valid && lse) {
+                // [B, Hq, Nq] (dense) or [Hq, total_q] (packed: Nq = total_q)
+                const long long li = varlen ? (long long)U.h * Nq + U.q_y0 + qi
+                                            : (long long)(U.b * Hq + U.h) * Nq + qi;
+                lse[li] = (Mx - kPShift + log2f(L)) * kLn2;
+            }
         }
         fav::setmaxnreg_inc<C::kRegLaunch>();
     } else {
@@ -518,7 +557,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 // ahead.
                 TileIt pf{0, 0, unit(0)};
                 for (int i = 0; i < C::kPrefetch; ++i) {
-                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
                     tile_next(pf);
                 }
                 const int early = min(KS, unit(0).n_kv);      // K tiles requested at the start
@@ -527,18 +566,18 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                     const int qb = k & 1;
                     if (unit_at(k + 1) >= 0) {
                         const Unit Un = unit(k + 1);
-                        fav::tma_prefetch_l2_5d(&tmQ, 0, Un.t * BM, 0, Un.h, Un.b);
+                        fav::tma_prefetch_l2_5d(&tmQ, 0, Un.q_y0 + Un.t * BM, 0, Un.h, Un.b);
                     }
                     // Q buffer qb was last read by unit k - 2's S MMAs (unit 0's Q: requested at the start)
                     if (k >= 2 && !fav::mbar_wait_il(q_empty + 8 * qb, ((k >> 1) - 1) & 1, status)) break;
                     if (k > 0) {
                         fav::mbar_arrive_expect_tx(q_full + 8 * qb, C::kQBytes);
-                        fav::tma_load_5d(sQ + qb * C::kQBytes, &tmQ, q_full + 8 * qb, 0, U.t * BM, 0, U.h, U.b);
+                        fav::tma_load_5d(sQ + qb * C::kQBytes, &tmQ, q_full + 8 * qb, 0, U.q_y0 + U.t * BM, 0, U.h, U.b);
                     }
                     for (int j = 0; j < U.n_kv; ++j, ++g) {
                         const int st = g % KS;
                         if (g < early) {
-                            if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                            if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
                             tile_next(pf);
                             continue;
                         }
@@ -547,11 +586,11 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                             break;
                         }
                         fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
-                        fav::tma_load_5d(sK + st * C::kKVBytes, &tmK, k_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
+                        fav::tma_load_5d(sK + st * C::kKVBytes, &tmK, k_full + 8 * st, 0, U.k_y0 + j * BN, 0, U.kvh, U.b);
     #ifdef FAV_TIMING
                         if (g < 32) tsk[g] = clock64();
     #endif
-                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
                         tile_next(pf);
                     }
                 }
@@ -568,21 +607,21 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 bool ok = true;
                 TileIt pf{0, 0, unit(0)};
                 for (int i = 0; i < C::kPrefetch; ++i) {
-                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
                     tile_next(pf);
                 }
                 for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
                     const Unit U = unit(k);
                     for (int j = 0; j < U.n_kv; ++j, ++g) {
                         const int st = g % VS;
-                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.j * BN, 0, pf.U.kvh, pf.U.b);
+                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
                         tile_next(pf);
                         if (g >= VS && !fav::mbar_wait_fast_il(v_empty + 8 * st, ((g / VS) - 1) & 1, status)) {
                             ok = false;
                             break;
                         }
                         fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
-                        fav::tma_load_5d(sV + st * C::kKVBytes, &tmV, v_full + 8 * st, 0, j * BN, 0, U.kvh, U.b);
+                        fav::tma_load_5d(sV + st * C::kKVBytes, &tmV, v_full + 8 * st, 0, U.k_y0 + j * BN, 0, U.kvh, U.b);
                     }
                 }
             }
@@ -594,9 +633,13 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                     const Unit U = unit(k);
                     const int qb = k & 1;
                     if (!fav::mbar_wait_il(o_staged + 8 * qb, (k >> 1) & 1, status)) break;
-                    fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.t * BM, 0, U.h, U.b);
-                    fav::bulk_commit_group();
-                    fav::bulk_wait_read_all();         // the buffer may take the next Q tile
+                    // (a partial tile of a packed sequence was written by the epilogue: rows past
+                    // its end belong to the next sequence)
+                    if (!(varlen && U.t * BM + BM > U.len_q)) {
+                        fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.q_y0 + U.t * BM, 0, U.h, U.b);
+                        fav::bulk_commit_group();
+                        fav::bulk_wait_read_all();     // the buffer may take the next Q tile
+                    }
                     fav::mbar_arrive(q_empty + 8 * qb);
                 }
                 fav::bulk_wait_all();
@@ -744,8 +787,10 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     if (warp == C::kMmaWarp) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
 }
 
+// vunits: the unit table of a packed variable-length batch (device, 2 int4 per unit), or null.
 template <typename T, int D, bool kV16>
-fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
+fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream,
+                  const int4 *vunits = nullptr, int n_vunits = 0) {
     using C = PrefillCfg<D>;
     const void *vsrc = a.v;
     FavStrides vstr = a.vs;
@@ -765,15 +810,16 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
         cudaSuccess)
         return FAV_ERR_CUDA;
     const int n_qtiles = (a.Nq + BM - 1) / BM;
-    const long long units = (long long)n_qtiles * a.B * a.Hq;
+    const long long units = vunits ? n_vunits : (long long)n_qtiles * a.B * a.Hq;
+    if (units <= 0) return FAV_OK;
     // (unit indices up to units + grid size are formed in int)
     if (units + a.num_sms > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
     // persistent: one CTA per SM at most, each working through its share of the units
     long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
     if (a.prefill_grid > 0) blocks = std::min<long long>(blocks, a.prefill_grid);
     kern<<<(unsigned)blocks, C::kThreads, C::kSmemBytes, stream>>>(
-        tmQ, tmK, tmV, tmO, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
-        a.scale * kLog2e, a.causal, a.dev_status);
+        tmQ, tmK, tmV, tmO, (T *)a.o, a.os, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv,
+        n_qtiles, a.scale * kLog2e, a.causal, a.dev_status, vunits, n_vunits);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_split_kernel", stream))
         return FAV_ERR_CUDA;
     return FAV_OK;
@@ -785,6 +831,13 @@ fav_status fav_launch_prefill_split(const FavArgs &a, void *workspace, cudaStrea
     if (a.D != 128) return FAV_ERR_UNSUPPORTED;
     return a.dtype == FAV_F16 ? launch<__half, 128, false>(a, workspace, s)
                               : launch<__nv_bfloat16, 128, true>(a, workspace, s);
+}
+
+fav_status fav_launch_prefill_varlen(const FavArgs &a, const int4 *units, int n_units,
+                                     void *workspace, cudaStream_t s) {
+    if (a.D != 128) return FAV_ERR_UNSUPPORTED;
+    return a.dtype == FAV_F16 ? launch<__half, 128, false>(a, workspace, s, units, n_units)
+                              : launch<__nv_bfloat16, 128, true>(a, workspace, s, units, n_units);
 }
 
 bool fav_prefill_supported(const FavArgs &a) {
