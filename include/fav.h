@@ -130,7 +130,7 @@ FAV_API fav_status fav_forward_strided(const void *q, const void *k, const void 
  *  cu_seqlens_k   cu_seqlens_q[b] .. cu_seqlens_q[b+1]-1 of q (keys likewise of k and v).  A
  *                 sequence with queries needs at least one key; causal (bottom-right aligned per
  *                 sequence) needs no more queries than keys; else FAV_ERR_INVALID_ARG.
- *  dtype, D       fp16 or bf16 with D = 128 (else FAV_ERR_UNSUPPORTED)
+ *  dtype, D       fp16 or bf16 with D = 64 or 128 (else FAV_ERR_UNSUPPORTED)
  *  other arguments as fav_forward.  The library builds the kernel's work list from the host
  *  arrays and copies it to a device buffer on `stream` (returning once the copy is staged);
  *  the call is otherwise asynchronous on `stream`.  total_q = 0 computes nothing.

@@ -316,34 +316,61 @@ fav_status fav_prefill_varlen(const void *q, const void *k, const void *v, void 
     fav_status st = validate_shape(1, Hq, Hkv, std::max(total_q, 1), std::max(total_k, 1), D,
                                    scale, 0, dtype);
     if (st != FAV_OK) return st;
-    if ((dtype != FAV_F16 && dtype != FAV_BF16) || D != 128) return FAV_ERR_UNSUPPORTED;
+    if ((dtype != FAV_F16 && dtype != FAV_BF16) || (D != 128 && D != 64)) return FAV_ERR_UNSUPPORTED;
     if (total_q == 0) return FAV_OK;                       // nothing to compute
+    auto key_tiles = [&](int t, int lq, int lk) {          // key tiles of query tile t
+        const int kv_end = causal ? std::min(lk, t * 128 + 128 + lk - lq) : lk;
+        return (kv_end + 127) / 128;
+    };
     // units: one 128-row query tile of one head of one sequence, heaviest causal work first
     // (then sequence, tile, head: the heads of a GQA group side by side), as in the dense kernel
-    struct U { int s, h, t, n_kv, q0, k0, lq, lk; };
+    // D = 64 (two-tile kernel): a unit is a pair of query tiles of one sequence -- tile t of
+    // heads (h, h+1) of one GQA group when the group size is even, else tiles (2p, 2p+1) of
+    // one head (a missing second tile has no key tiles).
+    struct U { int s, h0, h1, t0, t1, n0, n1, q0, k0, lq, lk; };
     std::vector<U> units;
+    const bool pair_heads = (Hq / Hkv) % 2 == 0;
     for (int b = 0; b < B; ++b) {
         const int lq = cu_seqlens_q[b + 1] - cu_seqlens_q[b];
         const int lk = cu_seqlens_k[b + 1] - cu_seqlens_k[b];
-        for (int t = 0; t * 128 < lq; ++t) {
-            const int kv_end = causal ? std::min(lk, t * 128 + 128 + lk - lq) : lk;
-            const int n_kv = (kv_end + 127) / 128;
-            for (int h = 0; h < Hq; ++h)
-                units.push_back(U{b, h, t, n_kv, cu_seqlens_q[b], cu_seqlens_k[b], lq, lk});
+        const int ntq = (lq + 127) / 128;
+        const int q0 = cu_seqlens_q[b], k0 = cu_seqlens_k[b];
+        if (D == 128) {
+            for (int t = 0; t < ntq; ++t)
+                for (int h = 0; h < Hq; ++h)
+                    units.push_back(U{b, h, h, t, t, key_tiles(t, lq, lk), 0, q0, k0, lq, lk});
+        } else if (pair_heads) {
+            for (int t = 0; t < ntq; ++t)
+                for (int h = 0; h < Hq; h += 2) {
+                    const int n = key_tiles(t, lq, lk);
+                    units.push_back(U{b, h, h + 1, t, t, n, n, q0, k0, lq, lk});
+                }
+        } else {
+            for (int t = 0; t < ntq; t += 2)
+                for (int h = 0; h < Hq; ++h)
+                    units.push_back(U{b, h, h, t, t + 1, key_tiles(t, lq, lk),
+                                      t + 1 < ntq ? key_tiles(t + 1, lq, lk) : 0, q0, k0, lq, lk});
         }
     }
     if (units.size() + 4096 > 0x7fffffffu) return FAV_ERR_UNSUPPORTED;
     std::stable_sort(units.begin(), units.end(), [](const U &x, const U &y) {
-        if (x.n_kv != y.n_kv) return x.n_kv > y.n_kv;
+        const int wx = std::max(x.n0, x.n1), wy = std::max(y.n0, y.n1);
+        if (wx != wy) return wx > wy;
         if (x.s != y.s) return x.s < y.s;
-        if (x.t != y.t) return x.t < y.t;
-        return x.h < y.h;
+        if (x.t0 != y.t0) return x.t0 < y.t0;
+        return x.h0 < y.h0;
     });
-    std::vector<int> table(units.size() * 8);
+    const int per = D == 128 ? 8 : 12;                     // ints per unit in the table
+    std::vector<int> table(units.size() * per);
     for (size_t i = 0; i < units.size(); ++i) {
         const U &u = units[i];
-        const int e[8] = {u.s, u.h, u.t, u.n_kv, u.q0, u.k0, u.lq, u.lk};
-        std::copy(e, e + 8, table.begin() + 8 * i);
+        if (D == 128) {
+            const int e[8] = {u.s, u.h0, u.t0, u.n0, u.q0, u.k0, u.lq, u.lk};
+            std::copy(e, e + 8, table.begin() + 8 * i);
+        } else {
+            const int e[12] = {u.s, u.h0, u.h1, u.t0, u.t1, u.n0, u.n1, u.q0, u.k0, u.lq, u.lk, 0};
+            std::copy(e, e + 12, table.begin() + 12 * i);
+        }
     }
     FavArgs a = make_args(q, k, v, o, lse, 1, Hq, Hkv, total_q, total_k, D, scale, causal, dtype);
     a.qs = a.os = FavStrides{(long long)total_q * Hq * D, (long long)D, (long long)Hq * D};
@@ -370,8 +397,10 @@ fav_status fav_prefill_varlen(const void *q, const void *k, const void *v, void 
         ws = ds->ws_pre;
     }
     if (st == FAV_OK)
-        st = fav_launch_prefill_varlen(a, static_cast<const int4 *>(ds->ws_units),
-                                       (int)units.size(), ws, s);
+        st = D == 128 ? fav_launch_prefill_varlen(a, static_cast<const int4 *>(ds->ws_units),
+                                                  (int)units.size(), ws, s)
+                      : fav_launch_prefill_pair_varlen(a, static_cast<const int4 *>(ds->ws_units),
+                                                       (int)units.size(), ws, s);
     if (st == FAV_OK) g_last_path.store(FAV_PATH_PREFILL);
     return st;
 }

@@ -69,6 +69,11 @@ fav_status fav_launch_prefill_pair(const FavArgs &a, void *workspace, cudaStream
 // {first query row, first key row, query length, key length}, heaviest causal work first.
 fav_status fav_launch_prefill_varlen(const FavArgs &a, const int4 *units, int n_units,
                                      void *workspace, cudaStream_t s);
+// The same for D = 64 (fav_prefill_pair.cu): three int4 per unit, a pair of query tiles of one
+// sequence: {sequence, head 0, head 1, tile 0}, {tile 1, key tiles 0, key tiles 1, first query
+// row}, {first key row, query length, key length, -}.
+fav_status fav_launch_prefill_pair_varlen(const FavArgs &a, const int4 *units, int n_units,
+                                          void *workspace, cudaStream_t s);
 fav_status fav_launch_prefill(const FavArgs &a, void *workspace, cudaStream_t s);
 
 // With FAV_DEBUG_SYNC=1 in the environment: synchronise `s` after a launch and report a

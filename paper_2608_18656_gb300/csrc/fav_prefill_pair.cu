@@ -131,7 +131,7 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                    const __grid_constant__ CUtensorMap tmV, T *__restrict__ o, FavStrides os,
                    float *__restrict__ lse, const float *__restrict__ v_scale, int B, int Hq,
                    int Hkv, int Nq, int Nkv, int n_qtiles, int pair_heads, float scale_log2,
-                   int causal, int *status) {
+                   int causal, int *status, const int4 *__restrict__ vunits, int n_vunits) {
     using C = PrefillCfg<D>;
     using TP = __half;    // type of the weights P and of V in shared memory (P.V MMA)
     constexpr int S = C::kStages;
@@ -162,10 +162,15 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     // consecutive query tiles of one head.  The CTA takes units c, 2P-1-c, 2P+c, 4P-1-c, ...
     // (P CTAs, "snake" order): with the units sorted by decreasing work, this evens out the
     // sums per CTA.
+    // Variable-length batches (vunits != null): units from a table built on the host (three
+    // int4 each: {sequence, h0, h1, t0}, {t1, key tiles 0, key tiles 1, first query row},
+    // {first key row, query length, key length, -}), Q/O and K/V viewed as [1, H, total, D].
     struct Unit {
-        int b, h[2], t[2], n_kv_tiles[2], n_kv, kvh, bkv;
+        int b, h[2], t[2], n_kv_tiles[2], n_kv, kvh, bkv, q_y0, k_y0, len_q, len_k;
     };
-    const int n_units = pair_heads ? n_qtiles * B * (Hq / 2) : ((n_qtiles + 1) / 2) * B * Hq;
+    const bool varlen = vunits != nullptr;
+    const int n_units = varlen ? n_vunits
+                               : pair_heads ? n_qtiles * B * (Hq / 2) : ((n_qtiles + 1) / 2) * B * Hq;
     auto unit_at = [&](int k) {   // the k-th unit of this CTA, or -1
         const int P = gridDim.x, c = blockIdx.x;
         const int u = k * P + ((k & 1) ? (P - 1 - c) : c);
@@ -173,6 +178,27 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     };
     auto make_unit = [&](int u) {
         Unit U;
+        if (varlen) {
+            const int4 a = vunits[3 * u], c = vunits[3 * u + 1], e = vunits[3 * u + 2];
+            U.b = 0;
+            U.h[0] = a.y;
+            U.h[1] = a.z;
+            U.t[0] = a.w;
+            U.t[1] = c.x;
+            U.n_kv_tiles[0] = c.y;
+            U.n_kv_tiles[1] = c.z;
+            U.q_y0 = c.w;
+            U.k_y0 = e.x;
+            U.len_q = e.y;
+            U.len_k = e.z;
+            U.kvh = U.h[0] / G;
+            U.bkv = U.kvh;
+            U.n_kv = max(U.n_kv_tiles[0], U.n_kv_tiles[1]);
+            return U;
+        }
+        U.q_y0 = U.k_y0 = 0;
+        U.len_q = Nq;
+        U.len_k = Nkv;
         if (pair_heads) {
             const int units = B * (Hq / 2);
             const int r = u % units;
@@ -262,7 +288,7 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
 #pragma unroll
                     for (int bx = 0; bx < C::kBoxes; ++bx)
                         fav::tma_load_4d(sbase + C::kOffQ + i * C::kQBytes + bx * BM * 128, &tmQ,
-                                         q_full + 8 * i, bx * 64, U.t[i] * BM, U.h[i], U.b);
+                                         q_full + 8 * i, bx * 64, U.q_y0 + U.t[i] * BM, U.h[i], U.b);
                 }
                 // Each stage has its own empty barriers (one commit per use, waited in order).
                 for (int j = 0; j < U.n_kv; ++j, ++g) {
@@ -273,13 +299,13 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
 #pragma unroll
                     for (int bx = 0; bx < C::kBoxes; ++bx)
                         fav::tma_load_4d(sK + st * C::kKVBytes + bx * BN * 128, &tmK, k_full + 8 * st,
-                                         bx * 64, j * BN, U.kvh, U.b);
+                                         bx * 64, U.k_y0 + j * BN, U.kvh, U.b);
                     if (g >= S && !fav::mbar_wait(v_empty + 8 * st, ph, status)) { ok = false; break; }
                     fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
 #pragma unroll
                     for (int bx = 0; bx < C::kBoxes; ++bx)
                         fav::tma_load_4d(sV + st * C::kKVBytes + bx * BN * 128, &tmV, v_full + 8 * st,
-                                         bx * 64, j * BN, U.kvh, U.b);
+                                         bx * 64, U.k_y0 + j * BN, U.kvh, U.b);
                 }
             }
         }
@@ -422,8 +448,9 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
             const int ti = U.t[i], hi = U.h[i];
             const int q0 = ti * BM;
             const int qi = q0 + row;                          // query index of this row
-            const int lim = causal ? min(Nkv, qi + off + 1) : Nkv;       // visible keys: [0, lim)
-            const int lim_tile = causal ? min(Nkv, q0 + off + 1) : Nkv;  // smallest lim in the tile
+            const int uoff = U.len_k - U.len_q;               // bottom-right causal offset
+            const int lim = causal ? min(U.len_k, qi + uoff + 1) : U.len_k;      // visible keys: [0, lim)
+            const int lim_tile = causal ? min(U.len_k, q0 + uoff + 1) : U.len_k; // smallest lim in the tile
             float m = -INFINITY, l = 0.f;
             for (int j = 0; j < n_mine; ++j) {
                 if (k == 0) FAV_STAMP(ts, j, 0);
@@ -564,8 +591,8 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
             fav::tc::fence_after();
             const float vsc = kV16 ? v_scale[U.bkv] : 1.f;     // V = v_scale * (fp16 copy)
             const float inv_l = vsc / l;
-            const bool valid = qi < Nq;
-            T *orow = o + U.b * os.b + hi * os.h + (long long)qi * os.n;
+            const bool valid = qi < U.len_q;
+            T *orow = o + U.b * os.b + hi * os.h + (long long)(U.q_y0 + qi) * os.n;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t v[32];
@@ -583,7 +610,12 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                     }
                 }
             }
-            if (valid && lse) lse[(long long)(U.b * Hq + hi) * Nq + qi] = (m - kPShift + log2f(l)) * kLn2;
+            if (valid && lse) {
+                // [B, Hq, Nq] (dense) or [Hq, total_q] (packed: Nq = total_q)
+                const long long li = varlen ? (long long)hi * Nq + U.q_y0 + qi
+                                            : (long long)(U.b * Hq + hi) * Nq + qi;
+                lse[li] = (m - kPShift + log2f(l)) * kLn2;
+            }
             fav::tc::fence_before();
         }
     }
@@ -594,8 +626,10 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
     if (warp == kMmaWarp) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
 }
 
+// vunits: the unit table of a packed variable-length batch (device, 3 int4 per unit), or null.
 template <typename T, int D, bool kV16>
-fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
+fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream,
+                  const int4 *vunits = nullptr, int n_vunits = 0) {
     using C = PrefillCfg<D>;
     const void *vsrc = a.v;
     FavStrides vstr = a.vs;
@@ -616,14 +650,17 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream) {
     const int n_qtiles = (a.Nq + BM - 1) / BM;
     const int G = a.Hq / a.Hkv;
     const int pair_heads = (G % 2 == 0) ? 1 : 0;
-    const long long units = pair_heads ? (long long)n_qtiles * a.B * (a.Hq / 2)
+    const long long units = vunits ? n_vunits
+                          : pair_heads ? (long long)n_qtiles * a.B * (a.Hq / 2)
                                        : (long long)((n_qtiles + 1) / 2) * a.B * a.Hq;
-    if (units > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
+    if (units <= 0) return FAV_OK;
+    if (units + a.num_sms > 0x7fffffffLL) return FAV_ERR_UNSUPPORTED;
     // persistent: one CTA per SM at most, each working through its share of the units
-    const long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
+    long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
+    if (a.prefill_grid > 0) blocks = std::min<long long>(blocks, a.prefill_grid);
     kern<<<(unsigned)blocks, kThreads, C::kSmemBytes, stream>>>(
         tmQ, tmK, tmV, (T *)a.o, a.os, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
-        pair_heads, a.scale * kLog2e, a.causal, a.dev_status);
+        pair_heads, a.scale * kLog2e, a.causal, a.dev_status, vunits, n_vunits);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_pair_kernel", stream))
         return FAV_ERR_CUDA;
     return FAV_OK;
@@ -635,4 +672,11 @@ fav_status fav_launch_prefill_pair(const FavArgs &a, void *workspace, cudaStream
     if (a.D != 64) return FAV_ERR_UNSUPPORTED;
     return a.dtype == FAV_F16 ? launch<__half, 64, false>(a, workspace, s)
                               : launch<__nv_bfloat16, 64, true>(a, workspace, s);
+}
+
+fav_status fav_launch_prefill_pair_varlen(const FavArgs &a, const int4 *units, int n_units,
+                                          void *workspace, cudaStream_t s) {
+    if (a.D != 64) return FAV_ERR_UNSUPPORTED;
+    return a.dtype == FAV_F16 ? launch<__half, 64, false>(a, workspace, s, units, n_units)
+                              : launch<__nv_bfloat16, 64, true>(a, workspace, s, units, n_units);
 }

@@ -36,7 +36,7 @@ def test_rejects_invalid_arguments(kw):
     assert call(**kw) == 1
 
 
-@pytest.mark.parametrize("kw", [dict(D=64), dict(D=256), dict(dtype=fav.F32)])
+@pytest.mark.parametrize("kw", [dict(D=96), dict(D=256), dict(dtype=fav.F32)])
 def test_rejects_unsupported(kw):
     assert call(**kw) == 2
 

@@ -54,44 +54,50 @@ def check(q, k, v, cq, ck, o, lse, dtype, causal, scale):
         assert np.abs(lse[:, cq[b]:cq[b + 1]] - rl[0]).max() <= LSE_TOL, "sequence %d: LSE" % b
 
 
+@pytest.mark.parametrize("D", [128, 64])
 @pytest.mark.parametrize("dtype", [I.F16, I.BF16])
 @pytest.mark.parametrize("causal", [False, True])
-def test_varlen_self_attention(dtype, causal):
+def test_varlen_self_attention(dtype, causal, D):
     lens = [1, 64, 127, 128, 129, 300, 513, 7]
-    q, k, v, cq, ck = packed(dtype, lens, lens, 8, 2, 128, seed=17 + causal + 2 * dtype)
-    scale = float(np.float32(1.0 / np.sqrt(128)))
+    q, k, v, cq, ck = packed(dtype, lens, lens, 8, 2, D, seed=17 + causal + 2 * dtype + D)
+    scale = float(np.float32(1.0 / np.sqrt(D)))
     o, lse = run(dtype, q, k, v, cq, ck, causal, scale)
     check(q, k, v, cq, ck, o, lse, dtype, causal, scale)
 
 
+@pytest.mark.parametrize("D", [128, 64])
 @pytest.mark.parametrize("causal", [False, True])
-def test_varlen_more_keys_than_queries(causal):
+def test_varlen_more_keys_than_queries(causal, D):
     """Chunked prefill: each sequence's new queries attend to a longer key prefix (bottom-right
     causal); a sequence with no queries in the middle of the batch."""
     lq, lk = [100, 0, 250, 33, 128], [500, 40, 250, 1000, 129]
-    q, k, v, cq, ck = packed(I.BF16, lq, lk, 4, 4, 128, seed=23 + causal)
+    q, k, v, cq, ck = packed(I.BF16, lq, lk, 4, 4, D, seed=23 + causal + D)
     scale = 0.07
     o, lse = run(I.BF16, q, k, v, cq, ck, causal, scale)
     check(q, k, v, cq, ck, o, lse, I.BF16, causal, scale)
 
 
+@pytest.mark.parametrize("D,Hq,Hkv", [(128, 6, 3), (64, 6, 3), (64, 8, 2), (64, 3, 1)])
 @pytest.mark.parametrize("grid", [1, 5])
-def test_varlen_many_units_per_block(grid):
+def test_varlen_many_units_per_block(grid, D, Hq, Hkv):
+    """Few blocks, many units each; at D = 64 both unit pairings (two heads of an even GQA
+    group, or two consecutive tiles of one head)."""
     fav.set_prefill_grid(grid)
     lens = [200, 129, 40, 300]
-    q, k, v, cq, ck = packed(I.F16, lens, lens, 6, 3, 128, seed=31 + grid)
-    scale = float(np.float32(1.0 / np.sqrt(128)))
+    q, k, v, cq, ck = packed(I.F16, lens, lens, Hq, Hkv, D, seed=31 + grid + D + Hq)
+    scale = float(np.float32(1.0 / np.sqrt(D)))
     o, lse = run(I.F16, q, k, v, cq, ck, True, scale)
     check(q, k, v, cq, ck, o, lse, I.F16, True, scale)
 
 
-def test_varlen_equals_dense_prefill_bitwise():
+@pytest.mark.parametrize("D", [128, 64])
+def test_varlen_equals_dense_prefill_bitwise(D):
     """A one-sequence batch runs the dense kernel's arithmetic on the same tiles: equal to
     fav_forward on the same sequence bit for bit (O and LSE)."""
     import torch
     lens = [777]
-    q, k, v, cq, ck = packed(I.F16, lens, lens, 8, 2, 128, seed=3)
-    scale = float(np.float32(1.0 / np.sqrt(128)))
+    q, k, v, cq, ck = packed(I.F16, lens, lens, 8, 2, D, seed=3 + D)
+    scale = float(np.float32(1.0 / np.sqrt(D)))
     o, lse = run(I.F16, q, k, v, cq, ck, True, scale)
     to = lambda a: to_device(I.to_storage(np.ascontiguousarray(a), I.F16), I.F16)
     od, ld = fav.forward(to(q.transpose(1, 0, 2)[None]), to(k.transpose(1, 0, 2)[None]),
