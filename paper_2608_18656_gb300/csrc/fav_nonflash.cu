@@ -1,0 +1,162 @@
+// fav_nonflash.cu -- the non-flash self-attention of the paper's Self-attention section, as an
+// in-library comparison point: the full score matrix is materialised.
+//
+//   S = scale * Q K^T      one batched GEMM per KV head (its G query heads stacked as the rows),
+//                          fp32 scores in a workspace [B * Hq, Nq, Nkv]
+//   P = softmax(S) (mask)  fav_nonflash_softmax_kernel: one block per query row, the row in
+//                          shared memory; the weights (rounded to the I/O type) overwrite the
+//                          first half of their own fp32 row, and LSE = max + log(sum)
+//   O = P V                a second batched GEMM per KV head
+//
+// The GEMMs are cuBLAS (cublasGemmStridedBatchedEx, fp32 accumulation), loaded on first use with
+// dlopen so that libfav itself does not depend on cuBLAS; without it the entry point returns
+// FAV_ERR_UNSUPPORTED.  The paper's point is that the fused (flash) form avoids writing and
+// reading the N x N scores; this path exists to measure that difference on this GPU.
+#include <cuda_runtime.h>
+#include <dlfcn.h>
+#include <math.h>
+
+#include <mutex>
+
+#include "fav_device.cuh"
+#include "fav_internal.h"
+
+namespace {
+
+// The few cuBLAS declarations used here (cublas_v2.h's types, restated as plain integers so
+// that this file builds without the header on the include path).
+using cublasHandle_t = void *;
+using cublasStatus_t = int;
+constexpr int kCublasOpN = 0, kCublasOpT = 1;
+constexpr int kCudaR32F = 0, kCudaR16F = 2, kCudaR16BF = 14;     // cudaDataType_t
+constexpr int kCublasCompute32F = 68;                           // cublasComputeType_t
+constexpr int kCublasGemmDefault = -1;                          // cublasGemmAlgo_t
+using CreateFn = cublasStatus_t (*)(cublasHandle_t *);
+using SetStreamFn = cublasStatus_t (*)(cublasHandle_t, cudaStream_t);
+// cublasGemmStridedBatchedEx(handle, transa, transb, m, n, k, alpha, A, Atype, lda, strideA,
+//                            B, Btype, ldb, strideB, beta, C, Ctype, ldc, strideC, batchCount,
+//                            computeType, algo)
+using GemmFn = cublasStatus_t (*)(cublasHandle_t, int, int, int, int, int, const void *,
+                                  const void *, int, int, long long, const void *, int, int,
+                                  long long, const void *, void *, int, int, long long, int, int,
+                                  int);
+
+struct Cublas {
+    bool ok = false;
+    cublasHandle_t handle[64] = {};
+    CreateFn create = nullptr;
+    SetStreamFn set_stream = nullptr;
+    GemmFn gemm = nullptr;
+};
+
+Cublas &cublas() {
+    static Cublas c;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        // the copy already in the process (loaded by the caller's framework), else the loader's
+        void *h = dlopen("libcublas.so.13", RTLD_NOW | RTLD_GLOBAL);
+        if (!h) h = dlopen("/usr/local/cuda/lib64/libcublas.so.13", RTLD_NOW | RTLD_GLOBAL);
+        if (!h) return;
+        c.create = reinterpret_cast<CreateFn>(dlsym(h, "cublasCreate_v2"));
+        c.set_stream = reinterpret_cast<SetStreamFn>(dlsym(h, "cublasSetStream_v2"));
+        c.gemm = reinterpret_cast<GemmFn>(dlsym(h, "cublasGemmStridedBatchedEx"));
+        c.ok = c.create && c.set_stream && c.gemm;
+    });
+    return c;
+}
+
+// One block per query row: the row's Nkv scores (fp32) in shared memory, the causal mask
+// (bottom-right: key j visible while j <= Nkv - Nq + i), maximum, sum of exponentials, then the
+// weights p_j = exp(s_j - max) / sum rounded to T over the first half of the row's bytes
+// (row stride in T elements: 2 * Nkv), and LSE = max + log(sum).
+template <typename T>
+__global__ void __launch_bounds__(256)
+fav_nonflash_softmax_kernel(float *__restrict__ s, float *__restrict__ lse, int Nq, int Nkv,
+                            int causal) {
+    extern __shared__ float row[];
+    __shared__ float red[8];
+    const long long r = blockIdx.x;
+    const int i = (int)(r % Nq);
+    const int lim = causal ? min(Nkv, Nkv - Nq + i + 1) : Nkv;      // visible keys [0, lim)
+    float *src = s + r * Nkv;
+    float mx = -INFINITY;
+    for (int j = threadIdx.x; j < Nkv; j += blockDim.x) {
+        const float x = j < lim ? src[j] : -INFINITY;
+        row[j] = x;
+        mx = fmaxf(mx, x);
+    }
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(~0u, mx, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+    __syncthreads();
+    mx = red[0];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) mx = fmaxf(mx, red[w]);
+    __syncthreads();
+    float sum = 0.f;
+    for (int j = threadIdx.x; j < Nkv; j += blockDim.x) {
+        const float e = (mx == -INFINITY) ? 0.f : expf(row[j] - mx);
+        row[j] = e;
+        sum += e;
+    }
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(~0u, sum, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sum;
+    __syncthreads();
+    sum = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) sum += red[w];
+    const float inv = sum > 0.f ? 1.f / sum : 0.f;
+    T *p = reinterpret_cast<T *>(src);          // every score of the row is in shared memory
+    for (int j = threadIdx.x; j < Nkv; j += blockDim.x) p[j] = fav::Elem<T>::from_f(row[j] * inv);
+    if (lse && threadIdx.x == 0) lse[r] = sum > 0.f ? mx + logf(sum) : -INFINITY;
+}
+
+}  // namespace
+
+size_t fav_nonflash_workspace_bytes(const FavArgs &a) {
+    return (size_t)a.B * a.Hq * a.Nq * a.Nkv * sizeof(float);
+}
+
+bool fav_nonflash_shape_ok(const FavArgs &a) {
+    if (a.dtype != FAV_F16 && a.dtype != FAV_BF16) return false;
+    const long long G = a.Hq / a.Hkv;
+    return a.Nkv <= 32768 && G * a.Nq * a.Nkv < (1LL << 31) &&
+           (long long)a.B * a.Hq * a.Nq <= 0x7fffffffLL;
+}
+
+bool fav_nonflash_available() { return cublas().ok; }
+
+fav_status fav_launch_nonflash(const FavArgs &a, void *workspace, cudaStream_t stream) {
+    Cublas &c = cublas();
+    if (!c.ok) return FAV_ERR_UNSUPPORTED;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return FAV_ERR_CUDA;
+    // one handle per device; the stream binding and the two GEMMs stay under the lock
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!c.handle[dev] && c.create(&c.handle[dev]) != 0) return FAV_ERR_CUDA;
+    if (c.set_stream(c.handle[dev], stream) != 0) return FAV_ERR_CUDA;
+    const int G = a.Hq / a.Hkv, N = a.Nq, Nk = a.Nkv, D = a.D, M = G * N;
+    const int batch = a.B * a.Hkv;
+    const int io = a.dtype == FAV_F16 ? kCudaR16F : kCudaR16BF;
+    float *S = static_cast<float *>(workspace);
+    const float alpha_s = a.scale, one = 1.f, zero = 0.f;
+    // S^T (Nk x M, column-major) = K (Nk x D) . Q^T (D x M): row-major S = Q K^T, per KV head
+    if (c.gemm(c.handle[dev], kCublasOpT, kCublasOpN, Nk, M, D, &alpha_s, a.k, io, D,
+               (long long)Nk * D, a.q, io, D, (long long)M * D, &zero, S, kCudaR32F, Nk,
+               (long long)M * Nk, batch, kCublasCompute32F, kCublasGemmDefault) != 0)
+        return FAV_ERR_CUDA;
+    const long long rows = (long long)a.B * a.Hq * N;
+    const size_t smem = (size_t)Nk * sizeof(float);
+    auto kern = a.dtype == FAV_F16 ? fav_nonflash_softmax_kernel<__half>
+                                   : fav_nonflash_softmax_kernel<__nv_bfloat16>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)(smem > 48 * 1024 ? smem : 48 * 1024)) != cudaSuccess)
+        return FAV_ERR_CUDA;
+    kern<<<(unsigned)rows, 256, smem, stream>>>(S, a.lse, N, Nk, a.causal);
+    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_nonflash_softmax_kernel", stream))
+        return FAV_ERR_CUDA;
+    // O^T (D x M) = V^T (D x Nk) . P^T (Nk x M); P rows are 2 * Nk elements apart (in place)
+    if (c.gemm(c.handle[dev], kCublasOpN, kCublasOpN, D, M, Nk, &one, a.v, io, D,
+               (long long)Nk * D, S, io, 2 * Nk, (long long)M * Nk * 2, &zero, a.o, io, D,
+               (long long)M * D, batch, kCublasCompute32F, kCublasGemmDefault) != 0)
+        return FAV_ERR_CUDA;
+    return FAV_OK;
+}

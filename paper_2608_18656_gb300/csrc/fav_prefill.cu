@@ -142,7 +142,9 @@ template <int D> struct PrefillCfg {
 // bf16 I/O (kV16): Q, K and O are bf16; V has been converted to fp16 (tmV, scaled per KV head
 // by v_scale^-1, a power of two) so that P.V runs with fp16 weights, and the epilogue multiplies
 // O back by v_scale.  fp16 I/O: tmV is V itself.
-template <typename T, int D, bool kV16>
+// kVarlen: the units come from the packed variable-length table `vunits` (the dense kernel
+// compiles without any of the per-sequence offsets, lengths and partial-tile stores).
+template <typename T, int D, bool kV16, bool kVarlen>
 __global__ void __launch_bounds__(PrefillCfg<D>::kThreads, 1)
 fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                          const __grid_constant__ CUtensorMap tmK,
@@ -186,7 +188,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     // Unit u: query tile t = n_qtiles - 1 - u / (B * Hq) of head (b, h) = u % (B * Hq), so the
     // heads of one GQA group (consecutive h) run side by side.  The CTA takes units c, 2P-1-c,
     // 2P+c, 4P-1-c, ... (P CTAs, "snake" order), which evens out the work per CTA.
-    // Variable-length batches (vunits != null): the units come from a table built on the host
+    // Variable-length batches (kVarlen): the units come from a table built on the host
     // (sorted the same way), Q/O are [1, Hq, total_q, D] and K/V [1, Hkv, total_k, D] views of
     // the packed tensors, and a unit's rows start at its sequence's offsets q_y0 / k_y0.
     // Unit: TMA batch coordinate b, head h, query tile t of its sequence, key tiles n_kv, KV head
@@ -194,7 +196,8 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     struct Unit {
         int b, h, t, n_kv, kvh, q_y0, k_y0, len_q, len_k;
     };
-    const bool varlen = vunits != nullptr;
+    constexpr bool varlen = kVarlen;
+    constexpr int kUnitInts = kVarlen ? 12 : 8;                 // ints per unit-table entry
     const int n_units = varlen ? n_vunits : n_qtiles * BH;
     auto unit_at = [&](int k) {   // the k-th unit of this CTA, or -1
         const int P = gridDim.x, c = blockIdx.x;
@@ -203,7 +206,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     };
     auto make_unit = [&](int u) {
         Unit U;
-        if (varlen) {
+        if constexpr (varlen) {
             const int4 a = vunits[2 * u], c = vunits[2 * u + 1];
             U.b = 0;
             U.h = a.y;
@@ -231,10 +234,16 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     // integer divisions would otherwise sit on the critical path at every unit switch).
     auto unit = [&](int k) {
         if (k < C::kUnitTab) {
-            const int *e = utab + 12 * k;
+            const int *e = utab + kUnitInts * k;
             Unit U;
             U.b = e[0]; U.h = e[1]; U.t = e[2]; U.n_kv = e[3]; U.kvh = e[4];
-            U.q_y0 = e[5]; U.k_y0 = e[6]; U.len_q = e[7]; U.len_k = e[8];
+            if constexpr (varlen) {
+                U.q_y0 = e[5]; U.k_y0 = e[6]; U.len_q = e[7]; U.len_k = e[8];
+            } else {
+                U.q_y0 = U.k_y0 = 0;
+                U.len_q = Nq;
+                U.len_k = Nkv;
+            }
             return U;
         }
         return make_unit(unit_at(k));
@@ -293,9 +302,11 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         const int u = unit_at(k);
         if (u < 0) break;
         const Unit U = make_unit(u);
-        int *e = utab + 12 * k;
+        int *e = utab + kUnitInts * k;
         e[0] = U.b; e[1] = U.h; e[2] = U.t; e[3] = U.n_kv; e[4] = U.kvh;
-        e[5] = U.q_y0; e[6] = U.k_y0; e[7] = U.len_q; e[8] = U.len_k;
+        if constexpr (varlen) {
+            e[5] = U.q_y0; e[6] = U.k_y0; e[7] = U.len_q; e[8] = U.len_k;
+        }
     }
 
 #ifdef FAV_TIMING
@@ -787,8 +798,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     if (warp == C::kMmaWarp) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
 }
 
-// vunits: the unit table of a packed variable-length batch (device, 2 int4 per unit), or null.
-template <typename T, int D, bool kV16>
+// vunits: the unit table of a packed variable-length batch (device, 2 int4 per unit), or null
+// (then kVarlen is false).
+template <typename T, int D, bool kV16, bool kVarlen = false>
 fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream,
                   const int4 *vunits = nullptr, int n_vunits = 0) {
     using C = PrefillCfg<D>;
@@ -805,7 +817,7 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream,
     if (st == FAV_OK) st = fav_make_tmap_tiles(&tmV, vsrc, D, a.Nkv, a.Hkv, a.B, vstr, BN);
     if (st == FAV_OK) st = fav_make_tmap_tiles(&tmO, a.o, D, a.Nq, a.Hq, a.B, a.os, BM);
     if (st != FAV_OK) return st;
-    auto kern = fav_prefill_split_kernel<T, D, kV16>;
+    auto kern = fav_prefill_split_kernel<T, D, kV16, kVarlen>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
         cudaSuccess)
         return FAV_ERR_CUDA;
@@ -836,8 +848,9 @@ fav_status fav_launch_prefill_split(const FavArgs &a, void *workspace, cudaStrea
 fav_status fav_launch_prefill_varlen(const FavArgs &a, const int4 *units, int n_units,
                                      void *workspace, cudaStream_t s) {
     if (a.D != 128) return FAV_ERR_UNSUPPORTED;
-    return a.dtype == FAV_F16 ? launch<__half, 128, false>(a, workspace, s, units, n_units)
-                              : launch<__nv_bfloat16, 128, true>(a, workspace, s, units, n_units);
+    return a.dtype == FAV_F16
+               ? launch<__half, 128, false, true>(a, workspace, s, units, n_units)
+               : launch<__nv_bfloat16, 128, true, true>(a, workspace, s, units, n_units);
 }
 
 bool fav_prefill_supported(const FavArgs &a) {
