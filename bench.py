@@ -8,7 +8,7 @@ The same JSON line also reports the other workloads of the measurement plan (GQA
 prefill with outliers; fp16 GQA and bf16 MQA decode with the split-KV combine, in KV GB/s).
 
 Timing: W warm-up steps, then K timed steps, each bracketed by CUDA events on the launching
-stream; L2 is flushed before every timed step by reading a 256 MiB buffer (outside the
+stream; L2 is flushed before every timed step by reading a 1 GiB buffer (outside the
 events; a read leaves no dirty lines whose write-back would compete with the timed kernel).  e2e = the same metric through the host-buffer C-ABI call fav_forward_host
 (pinned host inputs copied in, O and LSE copied out, every step).  cpu_baseline = the fp64
 oracle on the host cores on a bounded sample of the workload (rank 0, N=1 only).
@@ -45,6 +45,8 @@ def parse():
     ap.add_argument("--extra", default=None,
                     help="comma-separated indices of the extra workloads to time (default: all)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle cpu_baseline")
+    ap.add_argument("--no-nonflash", action="store_true",
+                    help="skip the non-fused comparison (materialised scores) on the headline")
     return ap.parse_args()
 
 
@@ -181,12 +183,14 @@ def launches_per_call(fav):
 def time_device(fn, steps, warmup, stream, dist):
     """Per-step CUDA-event times (ms) of `fn`, L2 flushed before each timed step.
 
-    The flush READS a 256 MiB buffer (twice the L2): it evicts the previous step's data and
+    The flush READS a 1 GiB buffer (eight times the L2): it evicts the previous step's data and
     leaves only clean lines behind.  (A write-based flush would leave ~126 MB of dirty lines
-    whose write-back then competes with the timed kernel's own HBM traffic.)
+    whose write-back then competes with the timed kernel's own HBM traffic.)  Its ~150 us of
+    device time also keeps the GPU behind the host, so that the host's enqueue time of the
+    step never shows up as idle time between the events.
     """
     import torch
-    flush = torch.ones(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
+    flush = torch.ones(1024 * 1024 * 1024, dtype=torch.uint8, device="cuda")
     sink = torch.empty((), dtype=torch.uint8, device="cuda")
     # Untimed ramp: keep the GPU busy for >= 0.2 s so that its clocks have left their idle
     # state before the warm-up steps proper (a short timed run otherwise starts at idle clocks).
@@ -345,6 +349,9 @@ def fav_arm(args, dist):
                                "roofline": {"bound": "tensor", "achieved": tf / dist.world,
                                             "peak": pk["tflops"], "unit": "TFLOP/s",
                                             "frac": tf / dist.world / pk["tflops"]}})
+    nonflash = None
+    if not args.no_nonflash:
+        nonflash = bench_nonflash(fav, w, x, args, stream, dist, ms)
     clocks = sampler.stop() if sampler else None
 
     value = job_rate(w.flops, ms * 1e-3, dist.world) / 1e12
@@ -376,7 +383,7 @@ def fav_arm(args, dist):
         "data": "synthetic (seeded N(0,1) Q/K, U(-1,1) V)",
         "config": {"workload": w.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv, "Nq": w.Nq,
                    "Nkv": w.Nkv, "D": w.D, "causal": w.causal, "path": path,
-                   "l2": "flushed before every timed step (256 MiB read, outside the events)",
+                   "l2": "flushed before every timed step (1 GiB read, outside the events)",
                    "parallelism": "replicas" if dist.world > 1 else "single GPU"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": pk["tflops"],
                      "unit": "TFLOP/s", "frac": achieved / pk["tflops"], "traffic": traffic,
@@ -386,17 +393,49 @@ def fav_arm(args, dist):
         "clocks": clocks,
         "cpu_baseline": cpu,
         "extra": extras,
+        "nonflash": nonflash,
     }
     if dist.rank == 0:
         print(json.dumps(line), flush=True)
     dist.close()
 
 
+def bench_nonflash(fav, w, x, args, stream, dist, fused_ms):
+    """The headline workload through fav_forward_nonflash (two cuBLAS GEMMs around this
+    library's masked softmax, the N x N scores in HBM): the non-fused comparison point."""
+    import torch
+    q, k, v = device_tensors(w, x)
+    o = torch.empty_like(q)
+    lse = torch.empty((w.B, w.Hq, w.Nq), dtype=torch.float32, device="cuda")
+    ws = torch.empty(fav.nonflash_workspace_size(w.B, w.Hq, w.Nq, w.Nkv), dtype=torch.uint8,
+                     device="cuda")
+
+    def step():
+        fav.forward_nonflash(q, k, v, causal=w.causal, scale=w.scale, out=o, lse_out=lse,
+                             workspace=ws, stream=stream)
+    try:
+        step()
+        torch.cuda.synchronize()
+    except fav.FavError as e:
+        return {"unavailable": str(e)}
+    steps = max(3, min(args.steps, 20))
+    times, _ = time_device(step, steps, max(3, args.warmup), stream, dist)
+    ms = dist.max(statistics.mean(times))
+    return {"workload": w.name, "value": job_rate(w.flops, ms * 1e-3, dist.world) / 1e12,
+            "unit": "TFLOP/s", "ms_per_step": ms, "steps": steps,
+            "fused_speedup": ms / fused_ms,
+            "scores_bytes": fav.nonflash_workspace_size(w.B, w.Hq, w.Nq, w.Nkv),
+            "kernels": "cuBLAS S = scale Q K^T (fp32 out), fav_nonflash_softmax_kernel, "
+                       "cuBLAS O = P V"}
+
+
 def kernel_hash():
+    """Hash of the sources the headline (prefill, D = 128) kernel is compiled from: the
+    traffic figure recorded under profiles/ is used only while they are unchanged."""
     import hashlib
     h = hashlib.sha256()
     src = os.path.join(ROOT, "paper_2608_18656_gb300", "csrc")
-    for f in sorted(os.listdir(src)):
+    for f in ("fav_prefill.cu", "fav_device.cuh", "fav_tc.cuh"):
         h.update(open(os.path.join(src, f), "rb").read())
     return h.hexdigest()[:16]
 

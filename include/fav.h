@@ -27,6 +27,8 @@
 #ifndef FAV_H
 #define FAV_H
 
+#include <stddef.h>
+
 #if defined(__GNUC__)
 #define FAV_API __attribute__((visibility("default")))
 #else
@@ -169,6 +171,29 @@ FAV_API fav_status fav_decode_paged(const void *q, const void *k_cache, const vo
                                     const int *seq_lens, int B, int Hq, int Hkv, int Nq,
                                     int max_pages, int page_size, int num_pages, int D,
                                     float scale, int causal, fav_dtype dtype, void *stream);
+
+/*
+ * fav_forward_nonflash -- the same attention computed the non-fused way, as a comparison point
+ * for the fused kernels (Background section, self-attention: the scores S = scale * Q K^T are
+ * materialised, the masked row softmax gives P, and O = P V).  Two cuBLAS GEMMs per call
+ * (batched over the KV heads of all batches; the G = Hq / Hkv query heads sharing a KV head are
+ * stacked as the rows of one GEMM) and one softmax kernel of this library, which also writes
+ * LSE.  P is rounded to the I/O type before P V, as on the fused tensor-core paths.
+ *
+ *  q, k, v, o, lse, B..dtype   as fav_forward; dtype fp16 or bf16 (else FAV_ERR_UNSUPPORTED)
+ *  workspace        device buffer of at least fav_nonflash_workspace_size(B, Hq, Nq, Nkv)
+ *                   bytes (the fp32 scores, then the weights in place), 16-byte aligned,
+ *                   caller-owned; else FAV_ERR_INVALID_ARG
+ *  workspace_bytes  its size in bytes
+ *  Nkv <= 32768 (a score row lives in shared memory) and (Hq / Hkv) * Nq * Nkv < 2^31, else
+ *  FAV_ERR_UNSUPPORTED.  cuBLAS (libcublas.so.13) is loaded on the first call; if it cannot
+ *  be loaded the call returns FAV_ERR_UNSUPPORTED.  Asynchronous on `stream`.
+ */
+FAV_API size_t fav_nonflash_workspace_size(int B, int Hq, int Nq, int Nkv);
+FAV_API fav_status fav_forward_nonflash(const void *q, const void *k, const void *v, void *o,
+                                        float *lse, int B, int Hq, int Hkv, int Nq, int Nkv,
+                                        int D, float scale, int causal, fav_dtype dtype,
+                                        void *workspace, size_t workspace_bytes, void *stream);
 
 /*
  * fav_forward_host -- the same operation on HOST buffers (end-to-end call).

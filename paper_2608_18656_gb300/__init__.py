@@ -7,7 +7,7 @@ CPU fallback: without the built library every call raises.
 import ctypes
 import os
 
-__all__ = ["forward", "forward_host", "decode_paged", "prefill_varlen", "Strides", "set_path", "last_path", "set_decode_splits",
+__all__ = ["forward", "forward_nonflash", "nonflash_workspace_size", "forward_host", "decode_paged", "prefill_varlen", "Strides", "set_path", "last_path", "set_decode_splits",
            "last_decode_splits", "set_prefill_grid", "device_status", "release_workspace", "library_path",
            "FavError", "F32", "F16", "BF16", "PATH_AUTO", "PATH_SIMT", "PATH_DECODE",
            "PATH_PREFILL"]
@@ -63,6 +63,11 @@ def lib():
         L.fav_prefill_varlen.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, ctypes.c_float,
                                          i, i, vp]
         L.fav_prefill_varlen.restype = i
+        L.fav_nonflash_workspace_size.argtypes = [i, i, i, i]
+        L.fav_nonflash_workspace_size.restype = ctypes.c_size_t
+        L.fav_forward_nonflash.argtypes = [vp, vp, vp, vp, vp, i, i, i, i, i, i, ctypes.c_float,
+                                           i, i, vp, ctypes.c_size_t, vp]
+        L.fav_forward_nonflash.restype = i
         L.fav_status_string.argtypes = [i]
         L.fav_status_string.restype = ctypes.c_char_p
         L.fav_get_last_device_status.argtypes = []
@@ -141,6 +146,48 @@ def forward(q, k, v, causal=False, scale=None, return_lse=True, out=None, lse_ou
                                            o.data_ptr(), lse_ptr, *sd, B, Hq, Hkv, Nq, Nkv, D,
                                            float(scale), int(bool(causal)), _dtype_code(q),
                                            s.cuda_stream)
+    _check(st)
+    return o, lse
+
+
+def nonflash_workspace_size(B, Hq, Nq, Nkv):
+    """Bytes of device workspace fav_forward_nonflash needs (fp32 scores of every head)."""
+    return lib().fav_nonflash_workspace_size(B, Hq, Nq, Nkv)
+
+
+def forward_nonflash(q, k, v, causal=False, scale=None, out=None, lse_out=None, workspace=None,
+                     stream=None):
+    """The non-fused attention (fav_forward_nonflash): S = scale Q K^T materialised in a
+    workspace, masked row softmax, O = P V.  Contiguous fp16/bf16 tensors q [B,Hq,Nq,D],
+    k/v [B,Hkv,Nkv,D].  ``workspace`` is a CUDA uint8 tensor of at least
+    nonflash_workspace_size(...) bytes (allocated per call if None).  Returns (o, lse)."""
+    import torch
+    for t in (q, k, v):
+        if not t.is_cuda or t.dim() != 4 or not t.is_contiguous():
+            raise ValueError("tensors must be contiguous 4-D CUDA tensors")
+    if k.dtype != q.dtype or v.dtype != q.dtype:
+        raise TypeError("q, k and v must share a dtype")
+    B, Hq, Nq, D = q.shape
+    Bk, Hkv, Nkv, Dk = k.shape
+    if tuple(v.shape) != tuple(k.shape) or Bk != B or Dk != D:
+        raise ValueError("shape mismatch between q, k and v")
+    if scale is None:
+        import numpy as np
+        scale = float(np.float32(1.0 / np.sqrt(D)))
+    o = out if out is not None else torch.empty(q.shape, dtype=q.dtype, device=q.device)
+    lse = lse_out if lse_out is not None else torch.empty((B, Hq, Nq), device=q.device,
+                                                          dtype=torch.float32)
+    if not o.is_contiguous() or not lse.is_contiguous():
+        raise ValueError("out and lse_out must be contiguous")
+    need = nonflash_workspace_size(B, Hq, Nq, Nkv)
+    ws = workspace if workspace is not None else torch.empty(need, dtype=torch.uint8,
+                                                             device=q.device)
+    s = stream if stream is not None else torch.cuda.current_stream(q.device)
+    with torch.cuda.device(q.device):
+        st = lib().fav_forward_nonflash(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(),
+                                        lse.data_ptr(), B, Hq, Hkv, Nq, Nkv, D, float(scale),
+                                        int(bool(causal)), _dtype_code(q), ws.data_ptr(),
+                                        ws.numel() * ws.element_size(), s.cuda_stream)
     _check(st)
     return o, lse
 

@@ -13,7 +13,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libfav.so")
 SOURCES = ["fav_api.cu", "fav_simt.cu", "fav_decode.cu", "fav_prefill.cu", "fav_prefill_pair.cu",
-           "fav_v16.cu", "fav_noalloc.cu"]
+           "fav_v16.cu", "fav_noalloc.cu", "fav_nonflash.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -43,7 +43,7 @@ def build(verbose=False, extra=()):
             if log:
                 sys.stderr.write(log)
     tmp = LIB + ".tmp.%d" % os.getpid()
-    cmd = [nvcc(), *ARCH, "-shared", "-cudart", "static", "-o", tmp] + [o for o, _ in results]
+    cmd = [nvcc(), *ARCH, "-shared", "-cudart", "static", "-ldl", "-o", tmp] + [o for o, _ in results]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError("link failed:\n%s%s" % (r.stdout, r.stderr))

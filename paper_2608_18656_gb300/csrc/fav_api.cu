@@ -501,6 +501,31 @@ fav_status fav_forward_strided(const void *q, const void *k, const void *v, void
     return forward_impl(a, static_cast<cudaStream_t>(stream));
 }
 
+size_t fav_nonflash_workspace_size(int B, int Hq, int Nq, int Nkv) {
+    if (B <= 0 || Hq <= 0 || Nq <= 0 || Nkv <= 0) return 0;
+    FavArgs a{};
+    a.B = B; a.Hq = Hq; a.Nq = Nq; a.Nkv = Nkv;
+    return fav_nonflash_workspace_bytes(a);
+}
+
+fav_status fav_forward_nonflash(const void *q, const void *k, const void *v, void *o, float *lse,
+                                int B, int Hq, int Hkv, int Nq, int Nkv, int D, float scale,
+                                int causal, fav_dtype dtype, void *workspace,
+                                size_t workspace_bytes, void *stream) {
+    if (!q || !k || !v || !o || !workspace) return FAV_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(o, 16) ||
+        !aligned(workspace, 16))
+        return FAV_ERR_INVALID_ARG;
+    if (lse && !aligned(lse, 4)) return FAV_ERR_INVALID_ARG;
+    fav_status st = validate_shape(B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    if (st != FAV_OK) return st;
+    const FavArgs a = make_args(q, k, v, o, lse, B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    if (!fav_nonflash_shape_ok(a)) return FAV_ERR_UNSUPPORTED;
+    if (workspace_bytes < fav_nonflash_workspace_bytes(a)) return FAV_ERR_INVALID_ARG;
+    if (!fav_nonflash_available()) return FAV_ERR_UNSUPPORTED;
+    return fav_launch_nonflash(a, workspace, static_cast<cudaStream_t>(stream));
+}
+
 fav_status fav_forward_host(const void *q, const void *k, const void *v, void *o, float *lse,
                             int B, int Hq, int Hkv, int Nq, int Nkv, int D, float scale,
                             int causal, fav_dtype dtype, void *stream) {

@@ -1,0 +1,71 @@
+"""fav_forward_nonflash (materialised scores, cuBLAS GEMMs + this library's softmax kernel)
+against the fp64 oracle on seeded inputs (needs a GB300)."""
+import numpy as np
+import pytest
+
+import paper_2608_18656_gb300 as fav
+from paper_2608_18656_gb300 import inputs as I
+import gpu_util
+from gpu_util import check, sample_rows, to_device
+
+pytestmark = pytest.mark.gpu
+
+
+def W(dtype, B, Hq, Hkv, Nq, Nkv, D, causal=False, outliers=False, seed=7):
+    return I.Workload("t", dtype, B, Hq, Hkv, Nq, Nkv, D, causal, outliers, seed)
+
+
+# Tolerance on O.  fp16: the library's 3e-3.  bf16: this path rounds the normalised weights P
+# to bf16 (8 significant bits, unit roundoff u = 2^-8) before P V, where the fused kernels use
+# fp16 weights; so |sum_j p_j d_j v_j| <= u max|v| with sum_j p_j = 1, plus the final rounding
+# of O to bf16, u |O| <= u max|v|: 2 * 2^-8 * max|v|, and every input here has |v| <= 1.
+NONFLASH_O_TOL = {I.F16: gpu_util.O_TOL[I.F16], I.BF16: 2.0 ** -7}
+
+
+@pytest.fixture(autouse=True)
+def _nonflash_tolerance(monkeypatch):
+    monkeypatch.setattr(gpu_util, "O_TOL", {**gpu_util.O_TOL, **NONFLASH_O_TOL})
+
+
+def run_nonflash(w, x, workspace=None):
+    import torch
+    q, k, v = (to_device(x[n + "_bits"], w.dtype) for n in ("q", "k", "v"))
+    o, lse = fav.forward_nonflash(q, k, v, causal=w.causal, scale=w.scale, workspace=workspace)
+    torch.cuda.synchronize()
+    return o.float().cpu().numpy().astype(np.float64), lse.cpu().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("dtype", [I.F16, I.BF16])
+@pytest.mark.parametrize("B,Hq,Hkv,Nq,Nkv,D,causal", [
+    (1, 4, 4, 128, 128, 128, True),        # MHA, one tile
+    (2, 8, 2, 300, 300, 64, True),         # GQA, ragged length
+    (1, 8, 1, 200, 517, 128, True),        # MQA, Nq < Nkv (bottom-right mask)
+    (2, 4, 2, 257, 1000, 128, False),
+    (1, 2, 2, 1, 333, 64, False),          # one query row
+    (1, 4, 2, 1, 1, 128, True),            # one key
+])
+def test_nonflash_matches_oracle(dtype, B, Hq, Hkv, Nq, Nkv, D, causal):
+    w = W(dtype, B, Hq, Hkv, Nq, Nkv, D, causal, seed=Nq + Nkv + D)
+    x = I.make_inputs(w)
+    o, lse = run_nonflash(w, x)
+    check(w, o, lse, x)
+
+
+def test_nonflash_outliers_and_caller_workspace():
+    """Large-magnitude scores (outlier rows) and a caller-given, oversized workspace."""
+    import torch
+    w = W(I.BF16, 1, 8, 2, 384, 384, 128, True, outliers=True, seed=3)
+    x = I.make_inputs(w)
+    ws = torch.empty(fav.nonflash_workspace_size(1, 8, 384, 384) + 4096, dtype=torch.uint8,
+                     device="cuda")
+    o, lse = run_nonflash(w, x, workspace=ws)
+    check(w, o, lse, x)
+
+
+@pytest.mark.parametrize("idx", [1, 2])
+def test_nonflash_prefill_workloads_sampled(idx):
+    """The measured prefill workloads at full size, on sampled rows."""
+    w = I.WORKLOADS[idx]
+    x = I.make_inputs(w)
+    o, lse = run_nonflash(w, x)
+    check(w, o, lse, x, rows=sample_rows(w, 2048, seed=idx))
