@@ -3,9 +3,10 @@
 //
 //   S = scale * Q K^T      one batched GEMM per KV head (its G query heads stacked as the rows),
 //                          fp32 scores in a workspace [B * Hq, Nq, Nkv]
-//   P = softmax(S) (mask)  fav_nonflash_softmax_kernel: one block per query row, the row in
-//                          shared memory; the weights (rounded to the I/O type) overwrite the
-//                          first half of their own fp32 row, and LSE = max + log(sum)
+//   P = softmax(S) (mask)  one block per query row, the row in registers (float4 loads; rows up
+//                          to 8192 keys, a multiple of 4) or else in shared memory; the weights
+//                          (rounded to the I/O type) overwrite the first half of their own fp32
+//                          row, and LSE = max + log(sum)
 //   O = P V                a second batched GEMM per KV head
 //
 // The GEMMs are cuBLAS (cublasGemmStridedBatchedEx, fp32 accumulation), loaded on first use with
@@ -108,6 +109,99 @@ fav_nonflash_softmax_kernel(float *__restrict__ s, float *__restrict__ lse, int 
     if (lse && threadIdx.x == 0) lse[r] = sum > 0.f ? mx + logf(sum) : -INFINITY;
 }
 
+// The same row softmax with the row in registers, for Nkv % 4 == 0 and Nkv <= 1024 * kVec:
+// each of the 256 threads holds kVec float4 of the row (16-byte loads; causal rows read only
+// their visible prefix), so the row is read once from HBM and the weights written once.
+template <typename T, int kVec>
+__global__ void __launch_bounds__(256)
+fav_nonflash_softmax_reg_kernel(float *__restrict__ s, float *__restrict__ lse, int Nq,
+                                int Nkv, int causal) {
+    __shared__ float red[2][8];
+    const long long r = blockIdx.x;
+    const int i = (int)(r % Nq);
+    const int lim = causal ? min(Nkv, Nkv - Nq + i + 1) : Nkv;      // visible keys [0, lim)
+    float *src = s + r * Nkv;
+    float4 x[kVec];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int v = 0; v < kVec; ++v) {
+        const int j = 4 * (v * 256 + (int)threadIdx.x);
+        float4 a = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+        if (j < lim) {
+            a = *reinterpret_cast<const float4 *>(src + j);
+            if (j + 1 >= lim) a.y = -INFINITY;
+            if (j + 2 >= lim) a.z = -INFINITY;
+            if (j + 3 >= lim) a.w = -INFINITY;
+        }
+        x[v] = a;
+        mx = fmaxf(mx, fmaxf(fmaxf(a.x, a.y), fmaxf(a.z, a.w)));
+    }
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(~0u, mx, o));
+    if ((threadIdx.x & 31) == 0) red[0][threadIdx.x >> 5] = mx;
+    __syncthreads();          // also: every thread has read its part of the row
+    mx = red[0][0];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) mx = fmaxf(mx, red[0][w]);
+    float sum = 0.f;
+#pragma unroll
+    for (int v = 0; v < kVec; ++v) {
+        float4 &a = x[v];
+        a.x = expf(a.x - mx);     // masked entries: exp(-inf) = 0 (mx is finite: lim >= 1)
+        a.y = expf(a.y - mx);
+        a.z = expf(a.z - mx);
+        a.w = expf(a.w - mx);
+        sum += (a.x + a.y) + (a.z + a.w);
+    }
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(~0u, sum, o);
+    if ((threadIdx.x & 31) == 0) red[1][threadIdx.x >> 5] = sum;
+    __syncthreads();
+    sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) sum += red[1][w];
+    const float inv = 1.f / sum;
+    T *p = reinterpret_cast<T *>(src);
+#pragma unroll
+    for (int v = 0; v < kVec; ++v) {
+        const int j = 4 * (v * 256 + (int)threadIdx.x);
+        if (j < Nkv) {
+            struct alignas(8) T4 { T a, b, c, d; } q;
+            q.a = fav::Elem<T>::from_f(x[v].x * inv);
+            q.b = fav::Elem<T>::from_f(x[v].y * inv);
+            q.c = fav::Elem<T>::from_f(x[v].z * inv);
+            q.d = fav::Elem<T>::from_f(x[v].w * inv);
+            *reinterpret_cast<T4 *>(p + j) = q;
+        }
+    }
+    if (lse && threadIdx.x == 0) lse[r] = mx + logf(sum);
+}
+
+// The softmax launch for I/O type T: registers when the row fits (and is 16-byte aligned),
+// shared memory otherwise.
+template <typename T>
+cudaError_t launch_softmax(float *S, float *lse, long long rows, int Nq, int Nk, int causal,
+                           cudaStream_t stream) {
+    const unsigned grid = (unsigned)rows;
+    if (Nk % 4 == 0 && Nk <= 8192) {
+        const int vec = (Nk + 1023) / 1024;
+        if (vec <= 1)
+            fav_nonflash_softmax_reg_kernel<T, 1><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
+        else if (vec <= 2)
+            fav_nonflash_softmax_reg_kernel<T, 2><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
+        else if (vec <= 4)
+            fav_nonflash_softmax_reg_kernel<T, 4><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
+        else
+            fav_nonflash_softmax_reg_kernel<T, 8><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
+        return cudaGetLastError();
+    }
+    const size_t smem = (size_t)Nk * sizeof(float);
+    auto kern = fav_nonflash_softmax_kernel<T>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)(smem > 48 * 1024 ? smem : 48 * 1024));
+    if (e != cudaSuccess) return e;
+    kern<<<grid, 256, smem, stream>>>(S, lse, Nq, Nk, causal);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 size_t fav_nonflash_workspace_bytes(const FavArgs &a) {
@@ -144,14 +238,10 @@ fav_status fav_launch_nonflash(const FavArgs &a, void *workspace, cudaStream_t s
                (long long)M * Nk, batch, kCublasCompute32F, kCublasGemmDefault) != 0)
         return FAV_ERR_CUDA;
     const long long rows = (long long)a.B * a.Hq * N;
-    const size_t smem = (size_t)Nk * sizeof(float);
-    auto kern = a.dtype == FAV_F16 ? fav_nonflash_softmax_kernel<__half>
-                                   : fav_nonflash_softmax_kernel<__nv_bfloat16>;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)(smem > 48 * 1024 ? smem : 48 * 1024)) != cudaSuccess)
-        return FAV_ERR_CUDA;
-    kern<<<(unsigned)rows, 256, smem, stream>>>(S, a.lse, N, Nk, a.causal);
-    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_nonflash_softmax_kernel", stream))
+    const cudaError_t e = a.dtype == FAV_F16
+                              ? launch_softmax<__half>(S, a.lse, rows, N, Nk, a.causal, stream)
+                              : launch_softmax<__nv_bfloat16>(S, a.lse, rows, N, Nk, a.causal, stream);
+    if (e != cudaSuccess || fav_debug_sync("fav_nonflash_softmax_kernel", stream))
         return FAV_ERR_CUDA;
     // O^T (D x M) = V^T (D x Nk) . P^T (Nk x M); P rows are 2 * Nk elements apart (in place)
     if (c.gemm(c.handle[dev], kCublasOpN, kCublasOpN, D, M, Nk, &one, a.v, io, D,

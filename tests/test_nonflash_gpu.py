@@ -43,8 +43,12 @@ def run_nonflash(w, x, workspace=None):
     (2, 4, 2, 257, 1000, 128, False),
     (1, 2, 2, 1, 333, 64, False),          # one query row
     (1, 4, 2, 1, 1, 128, True),            # one key
+    (1, 2, 1, 64, 6000, 64, True),         # row of 8 float4 per thread (registers)
+    (1, 2, 2, 16, 9000, 128, False),       # row longer than the register path (shared memory)
 ])
 def test_nonflash_matches_oracle(dtype, B, Hq, Hkv, Nq, Nkv, D, causal):
+    """Rows of 1..9000 keys: multiples of 4 up to 8192 take the register softmax, the others
+    the shared-memory one."""
     w = W(dtype, B, Hq, Hkv, Nq, Nkv, D, causal, seed=Nq + Nkv + D)
     x = I.make_inputs(w)
     o, lse = run_nonflash(w, x)
