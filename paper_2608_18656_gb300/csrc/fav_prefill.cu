@@ -366,13 +366,12 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 float s[SK];
                 // scores of this split from TMEM (and the mask: keys at or beyond lim get -inf)
                 {
-                    uint32_t r[SK / 32][32];
+                    static_assert(SK == 64, "one 64-column load per split");
+                    uint32_t r[SK];
+                    fav::tc::ld_32x32b_x64(trow + colS, r);
+                    fav::tc::wait_ld_dep(r);
 #pragma unroll
-                    for (int c = 0; c < SK / 32; ++c) fav::tc::ld_32x32b_x32(trow + colS + c * 32, r[c]);
-#pragma unroll
-                    for (int c = 0; c < SK / 32; ++c) fav::tc::wait_ld_dep(r[c]);
-#pragma unroll
-                    for (int c = 0; c < SK; ++c) s[c] = __uint_as_float(r[c >> 5][c & 31]);
+                    for (int c = 0; c < SK; ++c) s[c] = __uint_as_float(r[c]);
                     if (crosses) {
                         const int nvis = lim - key0;              // keys [0, nvis) of the split visible
 #pragma unroll

@@ -463,13 +463,13 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                 float s[BN];
                 // S row from TMEM (and the mask: keys at or beyond lim get -inf)
                 auto load_s = [&]() {
-                    uint32_t r[BN / 32][32];
+                    uint32_t r[BN / 64][64];
 #pragma unroll
-                    for (int c = 0; c < BN / 32; ++c) fav::tc::ld_32x32b_x32(trow + colS + c * 32, r[c]);
+                    for (int c = 0; c < BN / 64; ++c) fav::tc::ld_32x32b_x64(trow + colS + c * 64, r[c]);
 #pragma unroll
-                    for (int c = 0; c < BN / 32; ++c) fav::tc::wait_ld_dep(r[c]);
+                    for (int c = 0; c < BN / 64; ++c) fav::tc::wait_ld_dep(r[c]);
 #pragma unroll
-                    for (int c = 0; c < BN; ++c) s[c] = __uint_as_float(r[c >> 5][c & 31]);
+                    for (int c = 0; c < BN; ++c) s[c] = __uint_as_float(r[c >> 6][c & 63]);
                     if (crosses) {
 #pragma unroll
                         for (int c = 0; c < BN; ++c)
