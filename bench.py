@@ -173,10 +173,15 @@ def kv_bytes(w):
     return w.io_bytes
 
 
-def launches_per_call(fav):
+def launches_per_call(fav, w):
+    """libfav kernel launches per call: decode 1, plus the split merge (fav_combine_kernel)
+    with several splits; prefill 1, plus 2 for bf16 (the V conversion to fp16 and its
+    per-head scales)."""
     path = fav.last_path()
-    if path == fav.PATH_DECODE and fav.last_decode_splits() > 1:
-        return 2
+    if path == fav.PATH_DECODE:
+        return 2 if fav.last_decode_splits() > 1 else 1
+    if path == fav.PATH_PREFILL and w.dtype == I.BF16:
+        return 3
     return 1
 
 
@@ -318,7 +323,7 @@ def fav_arm(args, dist):
         torch.cuda.synchronize()
         if fav.device_status() != 0:
             raise RuntimeError("device wait timed out in %s" % w.name)
-        nl = launches_per_call(fav)
+        nl = launches_per_call(fav, w)
         path = fav.PATH_NAMES[fav.last_path()]
         times, wall = time_device(step, steps, warmup, stream, dist)
         ms = dist.max(statistics.mean(times))

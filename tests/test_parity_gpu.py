@@ -77,6 +77,18 @@ def test_decode_split_counts(splits):
     check(w, o, lse, x)
 
 
+def test_decode_split_counts_change_between_calls():
+    """Calls that alternate split counts on one shape (and one split in between) reuse the
+    split-KV workspace with different partial layouts: every call matches the oracle."""
+    w = W(I.BF16, 2, 16, 4, 1, 3000, 128, seed=21)
+    x = I.make_inputs(w)
+    for splits in (3, 7, 2, 7, 1, 5, 3):
+        fav.set_decode_splits(splits)
+        o, lse = run_gpu(w, x)
+        assert fav.last_path() == fav.PATH_DECODE
+        check(w, o, lse, x)
+
+
 @pytest.mark.parametrize("Nkv", [1, 2, 31, 32, 33, 63, 64, 65, 129])
 def test_decode_short_caches(Nkv):
     w = W(I.F16, 1, 4, 1, 1, Nkv, 128, seed=Nkv)
