@@ -9,15 +9,17 @@
 // pass over a K/V tile serves the whole group.
 //
 // Work decomposition: grid = (split, b * Hkv + g, 16-row chunk).  Each block streams its
-// range of 32-key tiles through a ring of shared-memory stages filled by TMA (one producer
-// warp, 128-byte swizzle), and four consumer warps take every fourth tile:
+// range of key tiles (32 keys at D = 128, 64 at D = 64) through a ring of shared-memory stages
+// filled by TMA (a K producer warp and a V producer warp, 128-byte swizzle); six consumer
+// warps own two ring stages each and take the tiles in turn:
 //   S = Q K^T (mma.sync, fp32 accumulate)  ->  mask (key >= Nkv; causal, bottom-right)
 //   -> online softmax in the exp2 domain (running max, rescale of O and l)
 //   -> O += P V with P rounded to the I/O type.
-// The four warp states are merged through shared memory; with one split the block writes O
-// and LSE directly, otherwise it writes the fp32 partial (O_s, lse_s) of its key range and
-// fav_combine_kernel merges them: L = logsumexp_s lse_s, O = sum_s exp(lse_s - L) O_s
-// (associativity of the online softmax of the paper's Algorithm "ggml-vec FlashAttention").
+// The consumer warp states are merged through shared memory; with one split the block writes
+// O and LSE directly, otherwise it writes the fp32 partial (O_s, lse_s) of its key range and
+// fav_combine_kernel (a programmatic dependent launch) merges them:
+// L = logsumexp_s lse_s, O = sum_s exp(lse_s - L) O_s (associativity of the online softmax of
+// the paper's Algorithm "ggml-vec FlashAttention").
 #include <cuda.h>
 #include <math.h>
 
