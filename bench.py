@@ -32,6 +32,7 @@ import numpy as np  # noqa: E402
 from paper_2608_18656_gb300 import inputs as I  # noqa: E402
 
 HEADLINE = 1          # index of the headline workload in inputs.WORKLOADS
+METRIC = "attention TFLOP/s (prefill) and KV GB/s (decode) on 1 GB300, % of roofline"
 EXTRA = [2, 3, 4]     # reported alongside
 
 
@@ -288,7 +289,7 @@ def reference_arm(args, dist):
     ms = statistics.mean(times) * 1e3
     value = flops / (ms * 1e-3) / 1e12
     sample = "%d of %d query rows of %s (seeded), fp64" % (len(rows), w.B * w.Hq * w.Nq, w.name)
-    line = {"impl": "reference", "metric": "attention TFLOP/s (prefill)", "value": value,
+    line = {"impl": "reference", "metric": METRIC, "value": value,
             "unit": "TFLOP/s", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -381,7 +382,7 @@ def fav_arm(args, dist):
         if tr and tr.get("kernel_source_hash") == kernel_hash():
             traffic = tr.get("dram_bytes_per_launch")
     line = {
-        "metric": "attention TFLOP/s (prefill) and KV GB/s (decode) on 1 GB300, % of roofline",
+        "metric": METRIC,
         "value": value, "unit": "TFLOP/s", "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": I.DTYPE_NAMES[w.dtype],
