@@ -152,8 +152,8 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                          const __grid_constant__ CUtensorMap tmO, T *__restrict__ o,
                          FavStrides os, float *__restrict__ lse,
                          const float *__restrict__ v_scale, int B, int Hq, int Hkv, int Nq,
-                         int Nkv, int n_qtiles, float scale_log2, int causal, int *status,
-                         const int4 *__restrict__ vunits, int n_vunits) {
+                         int Nkv, int n_qtiles, int head_block, float scale_log2, int causal,
+                         int *status, const int4 *__restrict__ vunits, int n_vunits) {
     using C = PrefillCfg<D>;
     using TP = __half;    // type of the weights P and of V in shared memory (P.V MMA)
     constexpr int KS = C::kKStages, VS = C::kVStages, NS = C::kSplits, SK = C::kSplitKeys;
@@ -185,9 +185,13 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     const int BH = B * Hq;
 
     // ---- work units: one query tile each, heaviest causal first ----
-    // Unit u: query tile t = n_qtiles - 1 - u / (B * Hq) of head (b, h) = u % (B * Hq), so the
-    // heads of one GQA group (consecutive h) run side by side.  The CTA takes units c, 2P-1-c,
-    // 2P+c, 4P-1-c, ... (P CTAs, "snake" order), which evens out the work per CTA.
+    // The B * Hq heads are taken in blocks of head_block heads (a multiple of the GQA group,
+    // chosen on the host so that a block's K and V fit in about half the L2); within a block,
+    // unit u is query tile t = n_qtiles - 1 - u / hb of head (b, h) = block start + u % hb
+    // (hb = the block's head count), so the heads of one GQA group (consecutive h) run side by
+    // side and a block's K/V tiles stay in L2 while all of its query tiles pass.  The CTA
+    // takes units c, 2P-1-c, 2P+c, 4P-1-c, ... (P CTAs, "snake" order), which evens out the
+    // work per CTA.
     // Variable-length batches (kVarlen): the units come from a table built on the host
     // (sorted the same way), Q/O are [1, Hq, total_q, D] and K/V [1, Hkv, total_k, D] views of
     // the packed tensors, and a unit's rows start at its sequence's offsets q_y0 / k_y0.
@@ -229,6 +233,17 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
         U.kvh = U.h / G;
         return U;
+    };
+    // With several head blocks (head_block < B * Hq; the host allows that only when every unit
+    // of a CTA fits the table below) unit u maps to the blocked order instead.
+    auto make_unit_blocked = [&](int u) {
+        if (varlen || head_block >= BH) return make_unit(u);
+        const int blk_units = n_qtiles * head_block;
+        const int blk = u / blk_units;
+        const int ul = u - blk * blk_units;
+        const int hb = min(head_block, BH - blk * head_block);
+        // the unit that the one-block order numbers (ul / hb) * BH + (head of this unit)
+        return make_unit((ul / hb) * BH + blk * head_block + ul % hb);
     };
     // The CTA's first kUnitTab units are computed once, in parallel, into shared memory (the
     // integer divisions would otherwise sit on the critical path at every unit switch).
@@ -290,7 +305,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         // TMEM allocation): they come from HBM and bound the time to the first scores.
         fav::tma_prefetch_desc(&tmQ);
         fav::tma_prefetch_desc(&tmK);
-        const Unit U0 = make_unit(unit_at(0));
+        const Unit U0 = make_unit_blocked(unit_at(0));
         fav::mbar_arrive_expect_tx(q_full, C::kQBytes);
         fav::tma_load_5d(sQ, &tmQ, q_full, 0, U0.q_y0 + U0.t * BM, 0, U0.h, U0.b);
         for (int g = 0; g < KS && g < U0.n_kv; ++g) {
@@ -301,7 +316,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     for (int k = threadIdx.x; k < C::kUnitTab; k += blockDim.x) {
         const int u = unit_at(k);
         if (u < 0) break;
-        const Unit U = make_unit(u);
+        const Unit U = make_unit_blocked(u);
         int *e = utab + kUnitInts * k;
         e[0] = U.b; e[1] = U.h; e[2] = U.t; e[3] = U.n_kv; e[4] = U.kvh;
         if constexpr (varlen) {
@@ -828,9 +843,19 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream,
     // persistent: one CTA per SM at most, each working through its share of the units
     long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
     if (a.prefill_grid > 0) blocks = std::min<long long>(blocks, a.prefill_grid);
+    // Heads per L2 block: K and V of head_block query heads (shared by the G heads of a group)
+    // within ~64 MB, a whole number of groups, at least one group and at most every head.  The
+    // blocked order is applied where the unit table is filled, so it needs every unit of a
+    // CTA in the table; otherwise one block.
+    const int G = a.Hq / a.Hkv;
+    const long long kv_bytes_group = 4LL * a.Nkv * D;             // K + V of one KV head
+    long long groups_per_block = std::max(1LL, (64LL << 20) / std::max(1LL, kv_bytes_group));
+    groups_per_block = std::min<long long>(groups_per_block, (long long)a.B * a.Hkv);
+    int head_block = (int)(groups_per_block * G);
+    if ((units + blocks - 1) / blocks > C::kUnitTab) head_block = a.B * a.Hq;
     kern<<<(unsigned)blocks, C::kThreads, C::kSmemBytes, stream>>>(
         tmQ, tmK, tmV, tmO, (T *)a.o, a.os, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv,
-        n_qtiles, a.scale * kLog2e, a.causal, a.dev_status, vunits, n_vunits);
+        n_qtiles, head_block, a.scale * kLog2e, a.causal, a.dev_status, vunits, n_vunits);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_split_kernel", stream))
         return FAV_ERR_CUDA;
     return FAV_OK;

@@ -6,7 +6,7 @@ import pytest
 
 import paper_2608_18656_gb300 as fav
 from paper_2608_18656_gb300 import inputs as I
-from gpu_util import LSE_TOL, O_TOL, check, run_gpu, sample_rows
+from gpu_util import LSE_TOL, O_TOL, check, run_gpu, sample_rows, to_device
 
 pytestmark = pytest.mark.gpu
 
@@ -228,6 +228,29 @@ def test_prefill_bf16_v_range(D):
         tol = np.where(mag > 0, 3e-3 * np.exp2(np.ceil(np.log2(np.maximum(mag, 1e-300)))), 0.0)
         assert (np.abs(o[0, h] - ref) <= tol).all(), "head %d" % h
     assert np.abs(lse - rl).max() <= LSE_TOL
+
+
+@pytest.mark.parametrize("dtype,B,Hq,Hkv,N", [
+    (I.F16, 3, 32, 32, 2048),     # 96 heads of 1 MB of K/V: blocks of 64 heads, the last of 32
+    (I.BF16, 4, 32, 8, 8192),     # 32 KV heads of 4 MB: blocks of 16 groups (64 query heads)
+])
+def test_prefill_head_blocks(dtype, B, Hq, Hkv, N):
+    """Heads taken in blocks whose K/V fit in L2 (query tiles of a block before the next
+    block): every query tile computed exactly once (output prefilled with NaN) and sampled rows
+    equal to the oracle."""
+    import torch
+    w = W(dtype, B, Hq, Hkv, N, N, 128, causal=True, seed=N + B)
+    x = I.make_inputs(w)
+    q, k, v = (to_device(x[n + "_bits"], dtype) for n in ("q", "k", "v"))
+    o = torch.full_like(q, float("nan"))
+    lse = torch.full((B, Hq, N), float("nan"), device="cuda")
+    fav.forward(q, k, v, causal=True, scale=w.scale, out=o, lse_out=lse)
+    torch.cuda.synchronize()
+    assert fav.device_status() == 0
+    assert fav.last_path() == fav.PATH_PREFILL
+    assert bool(torch.isfinite(o.float()).all()) and bool(torch.isfinite(lse).all())
+    o64 = o.float().cpu().numpy().astype(np.float64)
+    check(w, o64, lse.cpu().numpy().astype(np.float64), x, rows=sample_rows(w, 2048, seed=N))
 
 
 @pytest.mark.parametrize("grid", [1, 3, 7])
