@@ -10,7 +10,8 @@
 // come from L2).  On this GPU that becomes:
 //   * a unit is one 128-row query tile; the kernel is persistent (one CTA per SM at most) and
 //     CTA c works through units c, 2P-1-c, 2P+c, ... of the units sorted by decreasing causal
-//     work, with the next unit's Q tile loaded (TMA, 128-byte swizzle) into a second buffer;
+//     work within blocks of heads whose K/V fit in L2, with the next unit's Q tile loaded
+//     (TMA, 128-byte swizzle) into a second buffer;
 //   * 128-key K and V tiles are streamed by TMA (one copy instruction per tile) through rings
 //     of shared-memory stages;
 //   * S = Q K^T (M = 128, N = 128, K = 128) goes to one of two TMEM score buffers, so the
