@@ -436,13 +436,18 @@ def bench_nonflash(fav, w, x, args, stream, dist, fused_ms):
 
 
 def kernel_hash():
-    """Hash of the sources the headline (prefill, D = 128) kernel is compiled from: the
-    traffic figure recorded under profiles/ is used only while they are unchanged."""
+    """Hash of the code (comments and whitespace removed) of the sources the headline (prefill,
+    D = 128) kernel is compiled from: the traffic figure recorded under profiles/ is used only
+    while that code is unchanged."""
     import hashlib
+    import re
     h = hashlib.sha256()
     src = os.path.join(ROOT, "paper_2608_18656_gb300", "csrc")
     for f in ("fav_prefill.cu", "fav_device.cuh", "fav_tc.cuh"):
-        h.update(open(os.path.join(src, f), "rb").read())
+        text = open(os.path.join(src, f)).read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)      # block comments
+        text = re.sub(r"//[^\n]*", " ", text)                    # line comments
+        h.update(" ".join(text.split()).encode())
     return h.hexdigest()[:16]
 
 
