@@ -284,9 +284,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         (void)FAV_CHECK((sbase - raw_u32) + C::kOffTmemSlot + 4 <= fav::dynamic_smem_bytes(), status);
         for (int i = 0; i < 2; ++i) {
             fav::mbar_init(q_full + 8 * i, 1);
-            // last S commit + O store read; packed batches: the last S commit only (their O
-            // is written by the epilogue directly, not staged in the Q buffer)
-            fav::mbar_init(q_empty + 8 * i, varlen ? 1 : 2);
+            fav::mbar_init(q_empty + 8 * i, 2);          // last S commit + O store read
             fav::mbar_init(o_staged + 8 * i, 128);          // epilogue threads
             fav::mbar_init(xch_bar + 8 * i, C::kSoftWarps * 32);
             fav::mbar_init(s_full + 8 * i, 1);
@@ -519,11 +517,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             const float inv_l = vsc / L;
             const float a0 = w0 * inv_l, a1 = w1 * inv_l;
             const uint32_t stage = sQ + (k & 1) * C::kQBytes + row * 128;
-            // Packed batches write O row by row straight from here (a sequence's last tile has
-            // rows of the next sequence past its end, and short units must not wait for an O
-            // store before their Q buffer is reused: +12 % on prompts of 64-512 tokens); dense
-            // tiles go through the Q buffer and one TMA store (4 % faster on long sequences).
-            constexpr bool partial = varlen;
+            // the last tile of a packed sequence is written row by row (its rows past the end
+            // belong to the next sequence); every other tile goes through the TMA store
+            const bool partial = varlen && U.t * BM + BM > U.len_q;
             const bool valid = qi < U.len_q;
             T *orow = o + U.b * os.b + U.h * os.h + (long long)(U.q_y0 + qi) * os.n;
 #pragma unroll
@@ -558,10 +554,8 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             // O has been read: release it to the next unit's first P.V
             fav::tc::fence_before();
             fav::mbar_arrive(o_free);
-            if constexpr (!varlen) {
-                fav::tc::fence_proxy_async_smem();   // visible to the TMA store (async proxy)
-                fav::mbar_arrive(o_staged + 8 * (k & 1));
-            }
+            fav::tc::fence_proxy_async_smem();   // visible to the TMA store (async proxy)
+            fav::mbar_arrive(o_staged + 8 * (k & 1));
             if (valid && lse) {
                 // [B, Hq, Nq] (dense) or [Hq, total_q] (packed: Nq = total_q)
                 const long long li = varlen ? (long long)U.h * Nq + U.q_y0 + qi
@@ -659,15 +653,19 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             }
         } else if (warp == C::kStoreWarp) {
             // ---------------- O tiles: one TMA store per unit from its (free) Q buffer ----------------
-            if (lane == 0 && !varlen) {      // (packed batches: O written by the epilogue)
+            if (lane == 0) {
                 fav::tma_prefetch_desc(&tmO);
                 for (int k = 0, u; (u = unit_at(k)) >= 0; ++k) {
                     const Unit U = unit(k);
                     const int qb = k & 1;
                     if (!fav::mbar_wait_il(o_staged + 8 * qb, (k >> 1) & 1, status)) break;
-                    fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.t * BM, 0, U.h, U.b);
-                    fav::bulk_commit_group();
-                    fav::bulk_wait_read_all();     // the buffer may take the next Q tile
+                    // (a partial tile of a packed sequence was written by the epilogue: rows past
+                    // its end belong to the next sequence)
+                    if (!(varlen && U.t * BM + BM > U.len_q)) {
+                        fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.q_y0 + U.t * BM, 0, U.h, U.b);
+                        fav::bulk_commit_group();
+                        fav::bulk_wait_read_all();     // the buffer may take the next Q tile
+                    }
                     fav::mbar_arrive(q_empty + 8 * qb);
                 }
                 fav::bulk_wait_all();
