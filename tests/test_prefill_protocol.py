@@ -251,6 +251,23 @@ def test_protocol_never_stalls(B, Hq, Nq, Nkv, P):
             assert not stuck, "CTA %d of %d, units %s: %s" % (c, P, units, stuck)
 
 
+def test_protocol_random_shapes_and_grids():
+    """Random batch, head count, ragged lengths, causal or not, and grids from one block to one
+    block per query tile."""
+    rng = random.Random(2026)
+    for _ in range(40):
+        B, Hq = rng.randint(1, 3), rng.choice([1, 2, 3, 4, 8])
+        Nq = rng.randint(1, 700)
+        Nkv = Nq if rng.random() < 0.5 else rng.randint(Nq, 1200)
+        causal = rng.random() < 0.7
+        n_units = ((Nq + BM - 1) // BM) * B * Hq
+        P = rng.randint(1, n_units)
+        for c in rng.sample(range(P), min(P, 3)):
+            units = units_of(B, Hq, Nq, Nkv, P, c, causal)
+            stuck = simulate(units, random.Random(rng.random()))
+            assert not stuck, ((B, Hq, Nq, Nkv, causal, P, c), stuck)
+
+
 def test_planted_parity_mistake_is_caught():
     """The Q buffer's phase parity taken as ks % 2 instead of (ks / 2) % 2: in every run the MMA
     warp's wait for a unit's Q tile either passes before that tile has landed or, once it has,
