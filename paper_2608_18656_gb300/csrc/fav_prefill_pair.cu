@@ -367,8 +367,11 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                 // the offset carries over to the following key tiles.
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
-                    if (U.n_kv_tiles[i] == 0) continue;
+                    // Both Q copies are waited for, an unused tile's too: q_empty lets the
+                    // producer re-arm q_full for the next unit, which must not happen while this
+                    // unit's copy is still in flight (a second arrival in one phase).
                     if (!(ok = wait_all(q_full + 8 * i, k & 1))) break;
+                    if (U.n_kv_tiles[i] == 0) continue;
                     if (i == 1 && !(ok = wait_all(s_free, (nsi[0] - 1) & 1))) break;
                     if (nsi[i] > 0 && !(ok = wait_all(s_free + 8 * i, (nsi[i] - 1) & 1))) break;
                     fav::tc::fence_after();
