@@ -253,6 +253,22 @@ def test_prefill_head_blocks(dtype, B, Hq, Hkv, N):
     check(w, o64, lse.cpu().numpy().astype(np.float64), x, rows=sample_rows(w, 2048, seed=N))
 
 
+@pytest.mark.parametrize("grid", [0, 1, 2])
+@pytest.mark.parametrize("Nq,Nkv,causal", [(300, 64, False), (300, 300, True), (257, 257, True)])
+def test_prefill_pair_missing_second_tile(grid, Nq, Nkv, causal):
+    """D = 64 with an odd GQA group pairs query tiles (2p, 2p+1) of one head; with an odd number
+    of query tiles the last pair's second tile lies beyond the sequence (no key tiles, its Q copy
+    the zero fill).  Short caches make each unit's last S the first, so the Q buffers are handed
+    back to the producer almost at once."""
+    fav.set_path(fav.PATH_PREFILL)
+    w = W(I.BF16, 2, 3, 1, Nq, Nkv, 64, causal=causal, seed=Nq + Nkv + grid)
+    x = I.make_inputs(w)
+    fav.set_prefill_grid(grid)
+    o, lse = run_gpu(w, x)
+    assert fav.last_path() == fav.PATH_PREFILL
+    check(w, o, lse, x)
+
+
 @pytest.mark.parametrize("grid", [1, 3, 7])
 @pytest.mark.parametrize("dtype,D,causal,Hq,Hkv,N", [(I.F16, 128, True, 4, 2, 700),
                                                      (I.BF16, 64, True, 4, 1, 520),
