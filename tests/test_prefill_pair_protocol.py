@@ -255,3 +255,20 @@ def test_pair_protocol_random_shapes_and_grids():
             units = units_of(B, Hq, Hkv, Nq, Nkv, P, c, causal)
             stuck = simulate(units, random.Random(rng.random()))
             assert not stuck, ((B, Hq, Hkv, Nq, Nkv, causal, P, c), stuck)
+
+
+def test_pair_protocol_packed_batch_unit_orders():
+    """A packed variable-length batch gives a block any mix of units: pairs of heads (equal key
+    tiles), pairs of tiles of one sequence (the second with fewer or no key tiles), from short
+    and long sequences in the host's heaviest-first order."""
+    rng = random.Random(2608)
+    for _ in range(60):
+        units = []
+        for _ in range(rng.randint(1, 12)):
+            n0 = rng.randint(1, 9)
+            kind = rng.random()
+            n1 = n0 if kind < 0.4 else (0 if kind < 0.7 else rng.randint(1, n0 + 1))
+            units.append([n0, n1])
+        units.sort(key=lambda U: -max(U))
+        stuck = simulate(units, random.Random(rng.random()))
+        assert not stuck, (units, stuck)
