@@ -281,3 +281,14 @@ def test_planted_parity_mistake_is_caught():
             assert "passed q_full" in str(e)
         else:
             assert stuck and stuck["mma"][1].startswith("q_full")
+
+
+def test_protocol_packed_batch_unit_mixes():
+    """A packed variable-length batch gives a block units of any key-tile count (sequences of
+    different lengths, ragged last tiles) in the host's heaviest-first order."""
+    rng = random.Random(18656)
+    for _ in range(60):
+        units = [{"t": 0, "n_kv": rng.randint(1, 10)} for _ in range(rng.randint(1, 12))]
+        units.sort(key=lambda U: -U["n_kv"])
+        stuck = simulate(units, random.Random(rng.random()))
+        assert not stuck, (units, stuck)
