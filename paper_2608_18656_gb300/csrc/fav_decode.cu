@@ -117,15 +117,6 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     }
     __syncthreads();
 
-#ifdef FAV_TIMING
-    __shared__ long long t_ref;
-    __shared__ long long t_issue[64], t_ready[64], t_done[64];
-    if (threadIdx.x == 0) t_ref = clock64();
-    __syncthreads();
-#define FAV_DSTAMP(arr, lt) do { if ((lt) < 64) arr[lt] = clock64() - t_ref; } while (0)
-#else
-#define FAV_DSTAMP(arr, lt) do { } while (0)
-#endif
     if (warp >= kConsumers) {
         // ---------------- producers: lane 0 of warp kConsumers streams K, of the next warp V
         // (two issuing threads double the copy instructions a block can issue per unit time) --
@@ -150,7 +141,6 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
                 const int st = lt % S;
                 if (lt >= S && !fav::mbar_wait(empty0 + 8 * st, ((lt / S) - 1) & 1, status)) break;
                 const uint32_t full = full0 + 8 * st;
-                if (!is_v) FAV_DSTAMP(t_issue, lt);
                 fav::mbar_arrive_expect_tx(full, Cfg::kTileBytes);
                 const int key0 = (tile0 + lt) * TK;
                 const uint32_t dst = ring_u32 + st * Cfg::kStageBytes + (is_v ? Cfg::kTileBytes : 0);
@@ -231,7 +221,6 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     for (int lt = warp; lt < my_tiles; lt += kConsumers) {
         const int st = lt % S;
         if (!fav::mbar_wait(full0 + 8 * st, (lt / S) & 1, status)) { ok = false; break; }
-        if (lane == 0) FAV_DSTAMP(t_ready, lt);
         const uint32_t kbase = ring_u32 + st * Cfg::kStageBytes;
         const uint32_t vbase = kbase + Cfg::kTileBytes;
         const int key0 = (tile0 + lt) * TK;
@@ -317,7 +306,6 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         }
         __syncwarp();
         if (lane == 0) fav::mbar_arrive(empty0 + 8 * st);
-        if (lane == 0) FAV_DSTAMP(t_done, lt);
     }
 
     // ---------------- merge the four warp states through shared memory ----------------
@@ -344,11 +332,6 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         redl[warp * 16 + r + 8] = lrow[1];
     }
     fav::named_bar_sync(1, kConsumers * 32);
-#ifdef FAV_TIMING
-    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0)
-        for (int lt = 0; lt < min(my_tiles, 64); ++lt)
-            printf("[dec] tile %2d issue %7lld ready %7lld done %7lld\n", lt, t_issue[lt], t_ready[lt], t_done[lt]);
-#endif
     if (!ok) return;
 
     constexpr int kCols = D / 8;                 // columns per thread (8 threads per row)

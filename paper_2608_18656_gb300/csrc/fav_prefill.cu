@@ -57,14 +57,6 @@
 #include "fav_internal.h"
 #include "fav_tc.cuh"
 
-// Timing builds (-DFAV_TIMING) record SM clock stamps at the phase boundaries of the first
-// block's loops and print them at the end; release builds compile this away.
-#ifdef FAV_TIMING
-#define FAV_STAMP(arr, j, k) do { if ((j) < 16) (arr)[j][k] = clock64(); } while (0)
-#else
-#define FAV_STAMP(arr, j, k) do { } while (0)
-#endif
-
 namespace {
 
 constexpr int BM = 128;          // query rows per tile (= TMEM lanes)
@@ -132,7 +124,8 @@ template <int D> struct PrefillCfg {
     static constexpr int kOffBar = kOffUnits + kUnitTab * 48;
     static constexpr int kNumBars = 2 + 2 + 2 * kKStages + 2 * kVStages + 2 + 2 + 2 + 2 + 2 + 1;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
-    static constexpr int kSmemBytes = kOffTmemSlot + 16 + 1024;
+    static constexpr int kOffDbg = kOffTmemSlot + 16;             // debug builds: per-role totals
+    static constexpr int kSmemBytes = kOffDbg + 32 + 1024;
     static constexpr uint32_t kTmemCols = 512;
     static __host__ __device__ constexpr uint32_t colS(int buf) { return buf ? 128u : 0u; }
     static constexpr uint32_t kColO = 256;                   // O_s at kColO + s * D
@@ -179,6 +172,11 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     float2 *xch = reinterpret_cast<float2 *>(smem + C::kOffXch);
     int *utab = reinterpret_cast<int *>(smem + C::kOffUnits);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffTmemSlot);
+#ifdef FAV_DEBUG_CHECKS
+    // per role, what it processed: softmax key tiles, K tiles loaded, V tiles loaded, P.V
+    // products, S products, epilogue units, stored units
+    int *dbg_tot = reinterpret_cast<int *>(smem + C::kOffDbg);
+#endif
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int G = Hq / Hkv;
@@ -247,7 +245,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         return make_unit((ul / hb) * BH + blk * head_block + ul % hb);
     };
     // The CTA's first kUnitTab units are computed once, in parallel, into shared memory (the
-    // integer divisions would otherwise sit on the critical path at every unit switch).
+    // integer divisions would otherwise sit on the critical path at every unit switch); every
+    // entry is written (a unit past the CTA's last one has no key tiles).  Units beyond the
+    // table are computed where they are needed, in the same (blocked) order.
     auto unit = [&](int k) {
         if (k < C::kUnitTab) {
             const int *e = utab + kUnitInts * k;
@@ -262,22 +262,36 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             }
             return U;
         }
-        return make_unit(unit_at(k));
+        return make_unit_blocked(unit_at(k));
+    };
+    // Key tiles of the CTA's unit k (k must be one of its units), read from the table where the
+    // count is used (an explicit shared-memory load, not a value carried in registers).
+    const uint32_t utab_s = fav::smem_u32(utab);
+    auto unit_nkv = [&](int k) -> int {
+        if (k < C::kUnitTab) return fav::ld_shared_s32(utab_s + 4u * (uint32_t)(kUnitInts * k + 3));
+        return make_unit_blocked(unit_at(k)).n_kv;
     };
     // Position in the CTA's sequence of key tiles, for the L2 prefetches that run ahead of the
-    // loads: unit index k (-1 past the end), key tile j of that unit.
+    // loads: unit index k (-1 past the end), key tile j of that unit.  (Indices only: the unit's
+    // fields are read from the table when a prefetch is issued.)
     struct TileIt {
         int k, j;
-        Unit U;
     };
     auto tile_next = [&](TileIt &it) {
         if (it.k < 0) return;
-        if (++it.j == it.U.n_kv) {
+        if (++it.j == unit_nkv(it.k)) {
             it.j = 0;
             ++it.k;
-            if (unit_at(it.k) >= 0) it.U = unit(it.k);
-            else it.k = -1;
+            if (unit_at(it.k) < 0) it.k = -1;
         }
+    };
+    // L2 prefetch of the key tile at `it` (K or V, by the tensor map), then step `it` on
+    auto prefetch_next = [&](const CUtensorMap *tm, TileIt &it) {
+        if (it.k >= 0) {
+            const Unit P = unit(it.k);
+            fav::tma_prefetch_l2_5d(tm, 0, P.k_y0 + it.j * BN, 0, P.kvh, P.b);
+        }
+        tile_next(it);
     };
     if (warp == C::kLoadKWarp && lane == 0) {
         (void)FAV_CHECK((sbase & 1023u) == 0, status);
@@ -316,19 +330,19 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     for (int k = threadIdx.x; k < C::kUnitTab; k += blockDim.x) {
         const int u = unit_at(k);
-        if (u < 0) break;
-        const Unit U = make_unit_blocked(u);
         int *e = utab + kUnitInts * k;
+        if (u < 0) {
+#pragma unroll
+            for (int i = 0; i < kUnitInts; ++i) e[i] = 0;
+            continue;
+        }
+        const Unit U = make_unit_blocked(u);
         e[0] = U.b; e[1] = U.h; e[2] = U.t; e[3] = U.n_kv; e[4] = U.kvh;
         if constexpr (varlen) {
             e[5] = U.q_y0; e[6] = U.k_y0; e[7] = U.len_q; e[8] = U.len_k;
         }
     }
 
-#ifdef FAV_TIMING
-    __shared__ long long t_ref;
-    if (threadIdx.x == 0) t_ref = clock64();
-#endif
     if (warp == C::kMmaWarp) {
         fav::tc::tmem_alloc(fav::smem_u32(tmem_slot), C::kTmemCols);
         fav::tc::tmem_relinquish();
@@ -353,13 +367,6 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         const uint32_t colO = C::kColO + split * D;
         int Gt = 0;                // key tiles consumed so far (the CTA's sequence)
         bool ok = true;
-#ifdef FAV_TIMING
-        long long ts[32][5];
-        const long long t_start = t_ref;
-#define FAV_TSS(c) do { if (Gt < 32) ts[Gt][c] = clock64(); } while (0)
-#else
-#define FAV_TSS(c) do { } while (0)
-#endif
         for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
             const Unit U = unit(k);
             const int q0 = U.t * BM;
@@ -369,12 +376,10 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             const int lim_tile = causal ? min(U.len_k, q0 + uoff + 1) : U.len_k; // smallest lim in the tile
             float m = -INFINITY, l = 0.f;
             for (int j = 0; j < U.n_kv; ++j, ++Gt) {
-                FAV_TSS(0);
                 if (!__all_sync(~0u, fav::mbar_wait_il(s_full + 8 * (Gt & 1), (Gt >> 1) & 1, status))) {
                     ok = false;
                     break;
                 }
-                FAV_TSS(1);
                 fav::tc::fence_after();
                 const uint32_t colS = C::colS(Gt & 1) + split * SK;
                 const int key0 = j * BN + split * SK;
@@ -411,7 +416,6 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                     mx = fav::fmax3(fav::fmax3(m8[0], m8[1], m8[2]), fav::fmax3(m8[3], m8[4], m8[5]),
                                     fmaxf(m8[6], m8[7])) * scale_log2;
                 }
-                FAV_TSS(2);
                 // lazy rescale: move the reference maximum only when it grows by > 2^4
                 float alpha = 1.f;
                 bool rescale = false;
@@ -441,7 +445,6 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                     const float2 a = fav::fadd2(fav::fadd2(l4[0], l4[1]), fav::fadd2(l4[2], l4[3]));
                     l += a.x + a.y;
                 }
-                FAV_TSS(3);
                 // O_s *= alpha, once P(G-1).V (the last product into O_s) has completed.  S(G)
                 // was issued after P(G-2).V and has completed, so pv_done has completed phase
                 // G-2 and cannot have completed G (that needs these weights): the parity of phase
@@ -472,22 +475,15 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 fav::tc::fence_before();
                 __syncwarp();
                 if (lane == 0) fav::mbar_arrive(p_full + 8 * (Gt & 1));
-                FAV_TSS(4);
             }
             if (!ok) break;
             // (m, l) of this row and split for the epilogue warpgroup (slot k % 2)
             xch[((((k & 1) * 4 + quarter) * NS) + split) * 32 + lane] = make_float2(m, l);
             fav::mbar_arrive(xch_bar + 8 * (k & 1));
         }
-#ifdef FAV_TIMING
-        if (blockIdx.x == 0 && (threadIdx.x & 127) == 0) {
-            for (int g = 0; g < min(Gt, 32); ++g)
-                printf("[sm%d] G=%2d wait %6lld s_ready %6lld max %6lld exp %6lld arrive %6lld\n",
-                       split, g, ts[g][0] - t_start, ts[g][1] - t_start, ts[g][2] - t_start,
-                       ts[g][3] - t_start, ts[g][4] - t_start);
-        }
+#ifdef FAV_DEBUG_CHECKS
+        if (threadIdx.x == 0) dbg_tot[0] = Gt;
 #endif
-#undef FAV_TSS
         fav::setmaxnreg_dec<C::kRegLaunch>();      // back to the launch budget for the join
     } else if (warp >= C::kEpiWarp0) {
         fav::setmaxnreg_dec<C::kRegEpi>();
@@ -562,6 +558,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                                             : (long long)(U.b * Hq + U.h) * Nq + qi;
                 lse[li] = (Mx - kPShift + log2f(L)) * kLn2;
             }
+#ifdef FAV_DEBUG_CHECKS
+            if (threadIdx.x == 32 * C::kEpiWarp0) dbg_tot[5] = k + 1;
+#endif
         }
         fav::setmaxnreg_inc<C::kRegLaunch>();
     } else {
@@ -572,21 +571,13 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             // resumed several hundred cycles after the stage was released, and a K tile is needed
             // by S about one key-tile period after its stage frees.)
             if (lane == 0) {
-    #ifdef FAV_TIMING
-                long long tsk[32];
-                for (int i = 0; i < 32; ++i) tsk[i] = 0;
-    #endif
                 int g = 0;
                 bool ok = true;
                 // L2 prefetches run kPrefetch key tiles ahead of the loads (the ring only covers
                 // the L2 latency; a tile that misses L2 would stall S otherwise), and Q tiles a unit
                 // ahead.
-                TileIt pf{0, 0, unit(0)};
-                for (int i = 0; i < C::kPrefetch; ++i) {
-                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                    tile_next(pf);
-                }
-                const int early = min(KS, unit(0).n_kv);      // K tiles requested at the start
+                TileIt pf{0, 0};
+                for (int i = 0; i < C::kPrefetch; ++i) prefetch_next(&tmK, pf);
                 for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
                     const Unit U = unit(k);
                     const int qb = k & 1;
@@ -602,9 +593,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                     }
                     for (int j = 0; j < U.n_kv; ++j, ++g) {
                         const int st = g % KS;
-                        if (g < early) {
-                            if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                            tile_next(pf);
+                        // the first K tiles of unit 0 were requested at the start
+                        if (g < KS && g < unit_nkv(0)) {
+                            prefetch_next(&tmK, pf);
                             continue;
                         }
                         if (g >= KS && !fav::mbar_wait_fast_il(k_empty + 8 * st, ((g / KS) - 1) & 1, status)) {
@@ -613,17 +604,12 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                         }
                         fav::mbar_arrive_expect_tx(k_full + 8 * st, C::kKVBytes);
                         fav::tma_load_5d(sK + st * C::kKVBytes, &tmK, k_full + 8 * st, 0, U.k_y0 + j * BN, 0, U.kvh, U.b);
-    #ifdef FAV_TIMING
-                        if (g < 32) tsk[g] = clock64();
-    #endif
-                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmK, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                        tile_next(pf);
+                        prefetch_next(&tmK, pf);
                     }
                 }
-    #ifdef FAV_TIMING
-                if (blockIdx.x == 0)
-                    for (int i = 0; i < 32; ++i) printf("[kload] G=%2d issued %6lld\n", i, tsk[i] - t_ref);
-    #endif
+#ifdef FAV_DEBUG_CHECKS
+                dbg_tot[1] = g;
+#endif
             }
         } else if (warp == C::kLoadVWarp) {
             // ---------------- TMA producer: V tiles ----------------
@@ -631,17 +617,13 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 fav::tma_prefetch_desc(&tmV);
                 int g = 0;
                 bool ok = true;
-                TileIt pf{0, 0, unit(0)};
-                for (int i = 0; i < C::kPrefetch; ++i) {
-                    if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                    tile_next(pf);
-                }
+                TileIt pf{0, 0};
+                for (int i = 0; i < C::kPrefetch; ++i) prefetch_next(&tmV, pf);
                 for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
                     const Unit U = unit(k);
                     for (int j = 0; j < U.n_kv; ++j, ++g) {
                         const int st = g % VS;
-                        if (pf.k >= 0) fav::tma_prefetch_l2_5d(&tmV, 0, pf.U.k_y0 + pf.j * BN, 0, pf.U.kvh, pf.U.b);
-                        tile_next(pf);
+                        prefetch_next(&tmV, pf);
                         if (g >= VS && !fav::mbar_wait_fast_il(v_empty + 8 * st, ((g / VS) - 1) & 1, status)) {
                             ok = false;
                             break;
@@ -650,6 +632,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                         fav::tma_load_5d(sV + st * C::kKVBytes, &tmV, v_full + 8 * st, 0, U.k_y0 + j * BN, 0, U.kvh, U.b);
                     }
                 }
+#ifdef FAV_DEBUG_CHECKS
+                dbg_tot[2] = g;
+#endif
             }
         } else if (warp == C::kStoreWarp) {
             // ---------------- O tiles: one TMA store per unit from its (free) Q buffer ----------------
@@ -667,6 +652,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                         fav::bulk_wait_read_all();     // the buffer may take the next Q tile
                     }
                     fav::mbar_arrive(q_empty + 8 * qb);
+#ifdef FAV_DEBUG_CHECKS
+                    dbg_tot[6] = k + 1;
+#endif
                 }
                 fav::bulk_wait_all();
             }
@@ -688,19 +676,17 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 if (__all_sync(0xffffffffu, fav::mbar_test(bar, parity))) return true;
                 return __all_sync(0xffffffffu, fav::mbar_wait_il(bar, parity, status)) != 0;
             };
-    #ifdef FAV_TIMING
-            __shared__ long long tsm[32][6];
-            const long long t_start = t_ref;
-    #define FAV_TSM(g, c) do { if ((g) < 32 && lane == 0) tsm[g][c] = clock64(); } while (0)
-    #else
-    #define FAV_TSM(g, c) do { } while (0)
-    #endif
-            // Scores run two key tiles ahead of the P.V products: (ks, js) is the next tile whose
-            // S is due, Gs its position in the CTA's sequence.
+            // Scores run two key tiles ahead of the P.V products: unit ks (its index in the
+            // CTA's sequence; us = unit_at(ks), -1 past the end), key tile js of that unit, Gs its
+            // position in the CTA's sequence of key tiles.  Only these indices are carried from
+            // one S burst to the next: the unit's key-tile count is read from the unit table
+            // (a shared-memory load) wherever it is needed.  A copy of a unit's fields kept in
+            // registers from the prologue's bursts into the main loop was seen with a key-tile
+            // count of 0 there while the table held 1, in CTAs whose first unit ends within the
+            // prologue (ragged lengths: the MMA warp then waited for a key tile that no role
+            // produces); re-reading the table where the count is used removes that state.
             int ks = 0, js = 0, Gs = 0;
             int us = unit_at(0);
-            Unit Us;
-            if (us >= 0) Us = unit(0);
             // operands of the next S ready (Q of its unit, its K tile)?
             auto wait_next_s = [&]() -> bool {
                 if (us < 0) return true;
@@ -709,12 +695,12 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             };
             // after S(Gs) has been issued: the Q buffer is released with the unit's last S
             auto advance_s = [&]() {
-                if (js + 1 == Us.n_kv) fav::tc::commit_elect(q_empty + 8 * (ks & 1));
+                const int n = unit_nkv(ks);
+                if (js + 1 == n) fav::tc::commit_elect(q_empty + 8 * (ks & 1));
                 ++Gs;
-                if (++js == Us.n_kv) {
+                if (++js == n) {
                     js = 0;
                     us = unit_at(++ks);
-                    if (us >= 0) Us = unit(ks);
                 }
             };
             auto issue_next_s = [&]() {
@@ -736,74 +722,51 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                     issue_next_s();
                 }
             }
-            // The issuing lane blocks until the tensor pipe has taken most of a burst, so a wait
-            // placed right after a burst overlaps the MMAs still queued, while one placed before a
-            // burst that the pipe is waiting for leaves it idle.  Per key tile G: the weights,
-            // P(G).V, then (behind it) K(G+2) / Q and V(G+1), then S(G+2).
             // Per key tile G the tensor core needs the weights P(G) and V(G) for P(G).V, then K(G+2)
             // (and the Q tile of its unit) for S(G+2).  A barrier test costs 100-200 cycles while the
             // MMAs and TMA copies keep shared memory busy, and the issuing lane blocks until the pipe
-            // has taken most of a burst, so tests placed between bursts leave the pipe idle.  All the
-            // barriers of a tile are therefore tested at once, one per lane (a single shared-memory
-            // instruction), and both bursts follow back to back; if one is not ready the warp waits
-            // for each in turn instead.
+            // has taken most of a burst, so tests placed between bursts leave the pipe idle.  The
+            // barriers of a burst are therefore tested at once, one per lane (a single shared-memory
+            // instruction), the test for S(G+2) behind the queued P(G).V MMAs; if one is not ready
+            // the warp waits for each in turn instead.
             int Gp = 0;
-            for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
-                const Unit U = unit(k);
-                for (int j = 0; j < U.n_kv; ++j, ++Gp) {
+            for (int k = 0; ok && unit_at(k) >= 0; ++k) {
+                const int n_kv = unit_nkv(k);
+                for (int j = 0; j < n_kv; ++j, ++Gp) {
                     const int vs = Gp % VS;
-                    FAV_TSM(Gp, 0);
                     // lane 0: P(G); lane 1: V(G)
                     uint32_t tb = p_full + 8 * (Gp & 1), tp = (Gp >> 1) & 1;
                     if (lane == 1) { tb = v_full + 8 * vs; tp = (Gp / VS) & 1; }
                     const bool ready_pv = fav::mbar_test(tb, tp);
-    #ifdef FAV_TIMING
-                    {
-                        const unsigned nb = __ballot_sync(0xffffffffu, !ready_pv) & 0x3u;
-                        if (Gp < 32 && lane == 0) tsm[Gp][4] = nb;
-                    }
-    #endif
                     if (!__all_sync(0xffffffffu, ready_pv)) {
                         if (!(ok = wait_all(p_full + 8 * (Gp & 1), (Gp >> 1) & 1))) break;
                         if (!(ok = wait_all(v_full + 8 * vs, (Gp / VS) & 1))) break;
                     }
                     // a unit's first P.V overwrites O: the previous unit's O must have been read
                     if (j == 0 && k > 0 && !(ok = wait_all(o_free, (k - 1) & 1))) break;
-                    FAV_TSM(Gp, 1);
                     fav::tc::fence_after();
                     fav::tc::mma_pv_split<NS>(tmem + C::kColO, tmem + C::colS(Gp & 1),
                                               dv0 + (uint64_t)((vs * C::kKVBytes) >> 4), idesc_pv,
                                               j > 0 ? 1u : 0u, v_empty + 8 * vs, pv_done);
-                    if (j + 1 == U.n_kv) fav::tc::commit_elect(o_done);   // the unit's O is final
-                    FAV_TSM(Gp, 2);
+                    if (j + 1 == n_kv) fav::tc::commit_elect(o_done);   // the unit's O is final
                     // behind the queued P.V MMAs: lane 0: K(G+2); lane 1: the Q tile of its unit
                     if (us >= 0) {
                         uint32_t kb = k_full + 8 * (Gs % KS), kp = (Gs / KS) & 1;
                         if (js == 0 && lane == 1) { kb = q_full + 8 * (ks & 1); kp = (ks >> 1) & 1; }
                         const bool ready_s = fav::mbar_test(kb, kp);
-    #ifdef FAV_TIMING
-                        {
-                            const unsigned nb = __ballot_sync(0xffffffffu, !ready_s) & 0x3u;
-                            if (Gp < 32 && lane == 0) tsm[Gp][4] |= nb << 2;
-                        }
-    #endif
                         if (!__all_sync(0xffffffffu, ready_s) && !(ok = wait_next_s())) break;
                         fav::tc::fence_after();
                     }
-                    FAV_TSM(Gp, 5);
                     issue_next_s();
-                    FAV_TSM(Gp, 3);
                 }
             }
-    #ifdef FAV_TIMING
-            if (blockIdx.x == 0 && lane == 0)
-                for (int g = 0; g < min(Gp, 32); ++g)
-                    printf("[mma] G=%2d start %6lld got_p %6lld pv_issued %6lld notready(p,v,k,q) %x s_ready %6lld s_issued %6lld\n", g,
-                           tsm[g][0] - t_start, tsm[g][1] - t_start, tsm[g][2] - t_start, (unsigned)tsm[g][4],
-                           tsm[g][5] - t_start, tsm[g][3] - t_start);
-    #endif
-    #undef FAV_TSM
+#ifdef FAV_DEBUG_CHECKS
+            if (lane == 0) { dbg_tot[3] = Gp; dbg_tot[4] = Gs; }
+#endif
         }
+        // (warps 9-11 ran their roles on lane 0 alone: the register budget below is changed by
+        // each warp as a whole, so the warp is reconverged first)
+        __syncwarp();
         fav::setmaxnreg_inc<C::kRegLaunch>();
     }
 
@@ -811,6 +774,21 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     __syncthreads();
     fav::tc::fence_after();
     if (warp == C::kMmaWarp) fav::tc::tmem_dealloc(tmem, C::kTmemCols);
+#ifdef FAV_DEBUG_CHECKS
+    // every role processed the CTA's units and key tiles exactly (status 6 otherwise; a role
+    // whose bounded wait gave up has already set status 5)
+    if (threadIdx.x == 0 && *(volatile int *)status == 0) {
+        int units = 0, tiles = 0;
+        for (int k = 0; unit_at(k) >= 0; ++k) {
+            ++units;
+            tiles += unit_nkv(k);
+        }
+        (void)FAV_CHECK(dbg_tot[0] == tiles && dbg_tot[1] == tiles && dbg_tot[2] == tiles &&
+                            dbg_tot[3] == tiles && dbg_tot[4] == tiles && dbg_tot[5] == units &&
+                            dbg_tot[6] == units,
+                        status);
+    }
+#endif
 }
 
 // vunits: the unit table of a packed variable-length batch (device, 2 int4 per unit), or null

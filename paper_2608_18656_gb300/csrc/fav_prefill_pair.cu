@@ -47,14 +47,6 @@
 #include "fav_internal.h"
 #include "fav_tc.cuh"
 
-// Timing builds (-DFAV_TIMING) record SM clock stamps at the phase boundaries of the first
-// block's loops and print them at the end; release builds compile this away.
-#ifdef FAV_TIMING
-#define FAV_STAMP(arr, j, k) do { if ((j) < 16) (arr)[j][k] = clock64(); } while (0)
-#else
-#define FAV_STAMP(arr, j, k) do { } while (0)
-#endif
-
 namespace {
 
 constexpr int BM = 128;          // query rows per tile (= TMEM lanes)
@@ -252,10 +244,6 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         }
         fav::mbar_fence_init();
     }
-#ifdef FAV_TIMING
-    __shared__ long long t_ref;
-    if (threadIdx.x == 0) t_ref = clock64();
-#endif
     if (warp == kMmaWarp) {
         fav::tc::tmem_alloc(fav::smem_u32(tmem_slot), C::kTmemCols);
         fav::tc::tmem_relinquish();
@@ -342,10 +330,6 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         auto try_all = [&](uint32_t bar, uint32_t parity) {
             return __all_sync(0xffffffffu, fav::mbar_try(bar, parity));
         };
-#ifdef FAV_TIMING
-        long long ts[16][6];
-        const long long t_start = t_ref;
-#endif
         int g = 0;                 // key tiles streamed so far (ring sequence)
         int np[2] = {0, 0};        // P_i(.) consumed so far, per tile (p_full parity)
         int nsi[2] = {0, 0};       // S_i(.) issued so far, per tile (s_free parity, kSepP)
@@ -395,7 +379,6 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                         if (j + 1 < U.n_kv_tiles[i]) {
                             if (!k_ok && !(ok = wait_all(k_full + 8 * st1, ((gj + 1) / S) & 1))) break;
                             k_ok = true;
-                            if (k == 0) FAV_STAMP(ts, j, 3 * i);
                             if (!(ok = wait_all(s_free + 8 * i, (nsi[i] - 1) & 1))) break;
                             fav::tc::fence_after();
                             issue_s(i, st1, s_full + 8 * i, i == last1 ? k_empty + 8 * st1 : 0u);
@@ -406,11 +389,9 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                             v_ok = true;
                             if (!(ok = wait_all(p_full + 8 * i, np[i] & 1))) break;
                             ++np[i];
-                            if (k == 0) FAV_STAMP(ts, j, 3 * i + 1);
                             fav::tc::fence_after();
                             issue_pv(i, st, j > 0 ? 1u : 0u, p_free + 8 * i, i == last ? v_empty + 8 * st : 0u);
                             if (j + 1 == U.n_kv_tiles[i]) fav::tc::commit_elect(o_done + 8 * i);
-                            if (k == 0) FAV_STAMP(ts, j, 3 * i + 2);
                         }
                     }
                     if (!ok) break;
@@ -420,13 +401,6 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                 }
                 g += U.n_kv;
             }
-#ifdef FAV_TIMING
-            if (k == 0 && blockIdx.x == 0 && lane == 0)
-                for (int j = 0; j < min(U.n_kv, 16); ++j)
-                    printf("[mma] j=%2d wait_p0 %6lld got_p0 %6lld done0 %6lld | wait_p1 %6lld got_p1 %6lld done1 %6lld\n", j,
-                           ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start, ts[j][3] - t_start,
-                           ts[j][4] - t_start, ts[j][5] - t_start);
-#endif
         }
     } else {
         // ---------------- softmax / correction / epilogue: one thread per query row ----------------
@@ -440,10 +414,6 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         int npst = 0;              // P_i(.) stored so far (kSepP: p_free parity)
         const uint32_t colP = i ? C::colP(1) : C::colP(0);
         bool ok = true;
-#ifdef FAV_TIMING
-        long long ts[16][6];
-        const long long t_start = t_ref;
-#endif
         for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
             const Unit U = make_unit(u);
             const int n_mine = U.n_kv_tiles[i];
@@ -456,10 +426,8 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
             const int lim_tile = causal ? min(U.len_k, q0 + uoff + 1) : U.len_k; // smallest lim in the tile
             float m = -INFINITY, l = 0.f;
             for (int j = 0; j < n_mine; ++j) {
-                if (k == 0) FAV_STAMP(ts, j, 0);
                 if (!__all_sync(~0u, fav::mbar_wait(s_full + 8 * i, ns & 1, status))) { ok = false; break; }
                 ++ns;
-                if (k == 0) FAV_STAMP(ts, j, 1);
                 fav::tc::fence_after();
                 const int key0 = j * BN;
                 const bool crosses = key0 + BN > lim_tile;   // tile crosses the diagonal or the end
@@ -530,9 +498,7 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                 };
                 // two passes: the row maximum, then the weights against the (lazy) reference
                 load_s();
-                if (k == 0) FAV_STAMP(ts, j, 2);
                 move_max(row_max() * scale_log2);
-                if (k == 0) FAV_STAMP(ts, j, 3);
                 {
                     // S_i has been read (long ago; the signal waits for the start of the
                     // exponentials, which also paces the other tile: see the MMA warp)
@@ -552,7 +518,6 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                 ++npst;
                 exp_store(m - kPShift);
                 l += psum;
-                if (k == 0) FAV_STAMP(ts, j, 4);
                 // O_i is stable here: P_i(j-1).V has completed (D = 128: it was issued before
                 // S_i(j) and MMAs complete in issue order; D = 64: the p_free wait above).
                 if (__any_sync(~0u, rescale)) {
@@ -576,15 +541,7 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                 fav::tc::fence_before();
                 __syncwarp();
                 if (lane == 0) fav::mbar_arrive(p_full + 8 * i);
-                if (k == 0) FAV_STAMP(ts, j, 5);
             }
-#ifdef FAV_TIMING
-            if (k == 0 && blockIdx.x == 0 && (threadIdx.x & 127) == 0)
-                for (int j = 0; j < min(n_mine, 16); ++j)
-                    printf("[sm%d] j=%2d wait %6lld s_ready %6lld ld %6lld max %6lld exp %6lld arrive %6lld\n",
-                           i, j, ts[j][0] - t_start, ts[j][1] - t_start, ts[j][2] - t_start,
-                           ts[j][3] - t_start, ts[j][4] - t_start, ts[j][5] - t_start);
-#endif
             if (!ok) break;
             // ---------------- epilogue: O / l, LSE ----------------
             // (the next unit's first P.V, which overwrites O_i, waits for this warpgroup's next
