@@ -46,14 +46,6 @@ __device__ __forceinline__ uint64_t globaltimer() {
     return t;
 }
 
-// A 32-bit load from shared memory at the point where it is written (asm volatile: not merged
-// with earlier loads of the same word, not carried in a register from one use to the next).
-__device__ __forceinline__ int ld_shared_s32(uint32_t addr) {
-    int v;
-    asm volatile("ld.shared.s32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
-    return v;
-}
-
 // ---- mbarrier -------------------------------------------------------------------------
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");

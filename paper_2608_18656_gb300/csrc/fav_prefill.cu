@@ -247,7 +247,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     // The CTA's first kUnitTab units are computed once, in parallel, into shared memory (the
     // integer divisions would otherwise sit on the critical path at every unit switch); every
     // entry is written (a unit past the CTA's last one has no key tiles).  Units beyond the
-    // table are computed where they are needed, in the same (blocked) order.
+    // table are computed where they are needed: the host chooses the blocked order only when
+    // every unit of every CTA fits the table, so past it the plain order (make_unit) is the
+    // order the table would have held.
     auto unit = [&](int k) {
         if (k < C::kUnitTab) {
             const int *e = utab + kUnitInts * k;
@@ -262,35 +264,31 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             }
             return U;
         }
-        return make_unit_blocked(unit_at(k));
+        return make_unit(unit_at(k));
     };
-    // Key tiles of the CTA's unit k (k must be one of its units), read from the table where the
-    // count is used (an explicit shared-memory load, not a value carried in registers).
-    const uint32_t utab_s = fav::smem_u32(utab);
+    // Key tiles of the CTA's unit k (k must be one of its units).
     auto unit_nkv = [&](int k) -> int {
-        if (k < C::kUnitTab) return fav::ld_shared_s32(utab_s + 4u * (uint32_t)(kUnitInts * k + 3));
-        return make_unit_blocked(unit_at(k)).n_kv;
+        return k < C::kUnitTab ? utab[kUnitInts * k + 3] : make_unit(unit_at(k)).n_kv;
     };
     // Position in the CTA's sequence of key tiles, for the L2 prefetches that run ahead of the
-    // loads: unit index k (-1 past the end), key tile j of that unit.  (Indices only: the unit's
-    // fields are read from the table when a prefetch is issued.)
+    // loads (it steers prefetches only; the loads follow the unit table): unit index k (-1 past
+    // the end), key tile j of that unit.
     struct TileIt {
         int k, j;
+        Unit U;
     };
     auto tile_next = [&](TileIt &it) {
         if (it.k < 0) return;
-        if (++it.j == unit_nkv(it.k)) {
+        if (++it.j == it.U.n_kv) {
             it.j = 0;
             ++it.k;
-            if (unit_at(it.k) < 0) it.k = -1;
+            if (unit_at(it.k) >= 0) it.U = unit(it.k);
+            else it.k = -1;
         }
     };
     // L2 prefetch of the key tile at `it` (K or V, by the tensor map), then step `it` on
     auto prefetch_next = [&](const CUtensorMap *tm, TileIt &it) {
-        if (it.k >= 0) {
-            const Unit P = unit(it.k);
-            fav::tma_prefetch_l2_5d(tm, 0, P.k_y0 + it.j * BN, 0, P.kvh, P.b);
-        }
+        if (it.k >= 0) fav::tma_prefetch_l2_5d(tm, 0, it.U.k_y0 + it.j * BN, 0, it.U.kvh, it.U.b);
         tile_next(it);
     };
     if (warp == C::kLoadKWarp && lane == 0) {
@@ -576,8 +574,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 // L2 prefetches run kPrefetch key tiles ahead of the loads (the ring only covers
                 // the L2 latency; a tile that misses L2 would stall S otherwise), and Q tiles a unit
                 // ahead.
-                TileIt pf{0, 0};
+                TileIt pf{0, 0, unit(0)};
                 for (int i = 0; i < C::kPrefetch; ++i) prefetch_next(&tmK, pf);
+                const int early = min(KS, unit(0).n_kv);      // K tiles requested at the start
                 for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
                     const Unit U = unit(k);
                     const int qb = k & 1;
@@ -593,8 +592,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                     }
                     for (int j = 0; j < U.n_kv; ++j, ++g) {
                         const int st = g % KS;
-                        // the first K tiles of unit 0 were requested at the start
-                        if (g < KS && g < unit_nkv(0)) {
+                        if (g < early) {                // requested at the start
                             prefetch_next(&tmK, pf);
                             continue;
                         }
@@ -617,7 +615,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 fav::tma_prefetch_desc(&tmV);
                 int g = 0;
                 bool ok = true;
-                TileIt pf{0, 0};
+                TileIt pf{0, 0, unit(0)};
                 for (int i = 0; i < C::kPrefetch; ++i) prefetch_next(&tmV, pf);
                 for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
                     const Unit U = unit(k);
@@ -676,63 +674,23 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 if (__all_sync(0xffffffffu, fav::mbar_test(bar, parity))) return true;
                 return __all_sync(0xffffffffu, fav::mbar_wait_il(bar, parity, status)) != 0;
             };
-            // Scores run two key tiles ahead of the P.V products: unit ks (its index in the
-            // CTA's sequence; us = unit_at(ks), -1 past the end), key tile js of that unit, Gs its
-            // position in the CTA's sequence of key tiles.  Only these indices are carried from
-            // one S burst to the next: the unit's key-tile count is read from the unit table
-            // (a shared-memory load) wherever it is needed.  A copy of a unit's fields kept in
-            // registers from the prologue's bursts into the main loop was seen with a key-tile
-            // count of 0 there while the table held 1, in CTAs whose first unit ends within the
-            // prologue (ragged lengths: the MMA warp then waited for a key tile that no role
-            // produces); re-reading the table where the count is used removes that state.
+            // One flat loop: step t issues P(t-2).V (from t = 2 on) and then S(t), so the scores
+            // run two key tiles ahead of the P.V products.  Each side walks the CTA's units with
+            // its own indices (P.V: unit kp, key tile jp, count np; S: unit ks, key tile js,
+            // count ns, us = unit_at(ks) or -1 past the end), and reads a unit's key-tile count
+            // from the unit table when it moves on to that unit.  (One copy of each side's
+            // bookkeeping: an earlier form issued the first two S products in a separate
+            // prologue, and a unit count assigned there was seen as 0 in the main loop when the
+            // CTA's first unit ended within the prologue.)
             int ks = 0, js = 0, Gs = 0;
             int us = unit_at(0);
-            // operands of the next S ready (Q of its unit, its K tile)?
-            auto wait_next_s = [&]() -> bool {
-                if (us < 0) return true;
-                if (js == 0 && !wait_all(q_full + 8 * (ks & 1), (ks >> 1) & 1)) return false;
-                return wait_all(k_full + 8 * (Gs % KS), (Gs / KS) & 1);
-            };
-            // after S(Gs) has been issued: the Q buffer is released with the unit's last S
-            auto advance_s = [&]() {
-                const int n = unit_nkv(ks);
-                if (js + 1 == n) fav::tc::commit_elect(q_empty + 8 * (ks & 1));
-                ++Gs;
-                if (++js == n) {
-                    js = 0;
-                    us = unit_at(++ks);
-                }
-            };
-            auto issue_next_s = [&]() {
-                if (us < 0) return;                      // no further tile
-                const int qb = ks & 1, st = Gs % KS;
-                fav::tc::mma_ss_burst_k128<D / 16>(
-                    tmem + C::colS(Gs & 1), dq0 + (uint64_t)((qb * C::kQBytes) >> 4),
-                    dk0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_qk, 0u, s_full + 8 * (Gs & 1),
-                    k_empty + 8 * st);
-                advance_s();
-            };
-            bool ok = wait_next_s();
-            if (ok) {
-                fav::tc::fence_after();
-                issue_next_s();
-                ok = wait_next_s();
-                if (ok) {
-                    fav::tc::fence_after();
-                    issue_next_s();
-                }
-            }
-            // Per key tile G the tensor core needs the weights P(G) and V(G) for P(G).V, then K(G+2)
-            // (and the Q tile of its unit) for S(G+2).  A barrier test costs 100-200 cycles while the
-            // MMAs and TMA copies keep shared memory busy, and the issuing lane blocks until the pipe
-            // has taken most of a burst, so tests placed between bursts leave the pipe idle.  The
-            // barriers of a burst are therefore tested at once, one per lane (a single shared-memory
-            // instruction), the test for S(G+2) behind the queued P(G).V MMAs; if one is not ready
-            // the warp waits for each in turn instead.
-            int Gp = 0;
-            for (int k = 0; ok && unit_at(k) >= 0; ++k) {
-                const int n_kv = unit_nkv(k);
-                for (int j = 0; j < n_kv; ++j, ++Gp) {
+            int ns = us >= 0 ? unit_nkv(0) : 0;
+            int kp = 0, jp = 0, Gp = 0;
+            int np = ns;
+            bool ok = true;
+            for (int t = 0; ok; ++t) {
+                if (t >= 2) {
+                    if (unit_at(kp) < 0) break;          // every P.V has been issued
                     const int vs = Gp % VS;
                     // lane 0: P(G); lane 1: V(G)
                     uint32_t tb = p_full + 8 * (Gp & 1), tp = (Gp >> 1) & 1;
@@ -743,21 +701,46 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                         if (!(ok = wait_all(v_full + 8 * vs, (Gp / VS) & 1))) break;
                     }
                     // a unit's first P.V overwrites O: the previous unit's O must have been read
-                    if (j == 0 && k > 0 && !(ok = wait_all(o_free, (k - 1) & 1))) break;
+                    if (jp == 0 && kp > 0 && !(ok = wait_all(o_free, (kp - 1) & 1))) break;
                     fav::tc::fence_after();
                     fav::tc::mma_pv_split<NS>(tmem + C::kColO, tmem + C::colS(Gp & 1),
                                               dv0 + (uint64_t)((vs * C::kKVBytes) >> 4), idesc_pv,
-                                              j > 0 ? 1u : 0u, v_empty + 8 * vs, pv_done);
-                    if (j + 1 == n_kv) fav::tc::commit_elect(o_done);   // the unit's O is final
-                    // behind the queued P.V MMAs: lane 0: K(G+2); lane 1: the Q tile of its unit
-                    if (us >= 0) {
-                        uint32_t kb = k_full + 8 * (Gs % KS), kp = (Gs / KS) & 1;
-                        if (js == 0 && lane == 1) { kb = q_full + 8 * (ks & 1); kp = (ks >> 1) & 1; }
-                        const bool ready_s = fav::mbar_test(kb, kp);
-                        if (!__all_sync(0xffffffffu, ready_s) && !(ok = wait_next_s())) break;
-                        fav::tc::fence_after();
+                                              jp > 0 ? 1u : 0u, v_empty + 8 * vs, pv_done);
+                    if (jp + 1 == np) fav::tc::commit_elect(o_done);   // the unit's O is final
+                    ++Gp;
+                    if (++jp == np) {
+                        jp = 0;
+                        ++kp;
+                        np = unit_at(kp) >= 0 ? unit_nkv(kp) : 0;
                     }
-                    issue_next_s();
+                }
+                if (us < 0) continue;                    // no further S
+                // operands of S(Gs): its unit's Q tile (first key tile only) and K(Gs) -- tested
+                // at once (lane 0: K, lane 1: Q) behind the queued P.V MMAs
+                {
+                    uint32_t kb = k_full + 8 * (Gs % KS), kp_ = (Gs / KS) & 1;
+                    if (js == 0 && lane == 1) { kb = q_full + 8 * (ks & 1); kp_ = (ks >> 1) & 1; }
+                    const bool ready_s = fav::mbar_test(kb, kp_);
+                    if (!__all_sync(0xffffffffu, ready_s)) {
+                        if (js == 0 && !(ok = wait_all(q_full + 8 * (ks & 1), (ks >> 1) & 1))) break;
+                        if (!(ok = wait_all(k_full + 8 * (Gs % KS), (Gs / KS) & 1))) break;
+                    }
+                }
+                fav::tc::fence_after();
+                {
+                    const int qb = ks & 1, st = Gs % KS;
+                    fav::tc::mma_ss_burst_k128<D / 16>(
+                        tmem + C::colS(Gs & 1), dq0 + (uint64_t)((qb * C::kQBytes) >> 4),
+                        dk0 + (uint64_t)((st * C::kKVBytes) >> 4), idesc_qk, 0u,
+                        s_full + 8 * (Gs & 1), k_empty + 8 * st);
+                }
+                // the Q buffer is released with the unit's last S
+                if (js + 1 == ns) fav::tc::commit_elect(q_empty + 8 * (ks & 1));
+                ++Gs;
+                if (++js == ns) {
+                    js = 0;
+                    us = unit_at(++ks);
+                    ns = us >= 0 ? unit_nkv(ks) : 0;
                 }
             }
 #ifdef FAV_DEBUG_CHECKS

@@ -2,13 +2,14 @@
 (needs a GB300).
 
 These shapes give every block a first unit whose key tiles are all issued by the MMA warp's
-prologue (at most two key tiles), followed by short units: the length is not a multiple of the
-128-row tile, so the last query tile is partial and the heaviest unit has two key tiles.  With
-the key-tile count of such a unit carried in registers from the prologue into the main loop,
-the MMA warp of the D = 128 kernel saw a count of 0 and waited for a key tile that no role
-produces (the blocks' bounded waits gave up after 2 s and the call reported
-FAV_ERR_DEVICE_TIMEOUT).  Every case here compares every output row with the oracle and checks
-that no bounded wait gave up (run_gpu asserts a zero device status)."""
+first two S products (at most two key tiles), followed by short units: the length is not a
+multiple of the 128-row tile, so the last query tile is partial and the heaviest unit has two
+key tiles.  When the MMA warp issued those first two S products from a separate prologue, the
+key-tile count it took over from there for the block's second unit was 0 in the main loop, and
+the warp waited for a key tile that no role produces (the blocks' bounded waits gave up after
+2 s and the call reported FAV_ERR_DEVICE_TIMEOUT).  Every case here compares every output row
+with the oracle and checks that no bounded wait gave up (run_gpu asserts a zero device
+status)."""
 import numpy as np
 import pytest
 
