@@ -47,7 +47,11 @@ typedef enum {
     FAV_ERR_UNSUPPORTED = 2,    /* valid attention problem that no kernel here implements     */
     FAV_ERR_CUDA = 3,           /* a CUDA runtime call or kernel launch failed                */
     FAV_ERR_NO_MEMORY = 4,      /* the internal workspace could not be allocated              */
-    FAV_ERR_DEVICE_TIMEOUT = 5  /* a bounded wait inside a kernel ran out (see below)         */
+    FAV_ERR_DEVICE_TIMEOUT = 5, /* a bounded wait inside a kernel ran out (see below)         */
+    FAV_ERR_DEVICE_CHECK = 6,   /* a check of the self-checking -DFAV_DEBUG_CHECKS build failed
+                                   (an access it would have made was skipped)                 */
+    FAV_ERR_BAD_PAGE = 7        /* fav_decode_paged met a block-table entry outside
+                                   [0, num_pages): that page's keys were left out             */
 } fav_status;
 
 /* Kernel families (for fav_set_path / fav_last_path). */
@@ -153,8 +157,11 @@ FAV_API fav_status fav_prefill_varlen(const void *q, const void *k, const void *
  *  v_cache      token side by side), `dtype`, 16-byte aligned
  *  block_table  device int32 [B, max_pages]: key n of sequence b is row n % page_size of page
  *               block_table[b * max_pages + n / page_size].  Pages may be shared between
- *               sequences.  Entries past a sequence's length are not read; a page id outside
- *               [0, num_pages) reads as zeros.
+ *               sequences.  Entries past a sequence's length are not read.  An entry inside
+ *               a sequence's length that lies outside [0, num_pages) is not dereferenced:
+ *               that page's keys take no part in the softmax (a row with no other key gets
+ *               O = 0, LSE = -inf) and the kernel sets FAV_ERR_BAD_PAGE in the device status
+ *               word, which fav_get_last_device_status() reports.
  *  seq_lens     device int32 [B]: keys of each sequence, clamped to [0, max_pages * page_size]
  *  lse          device [B, Hq, Nq] fp32, or NULL
  *  page_size    a power of two in [16, 65536] (else FAV_ERR_UNSUPPORTED)
@@ -178,7 +185,10 @@ FAV_API fav_status fav_decode_paged(const void *q, const void *k_cache, const vo
  * materialised, the masked row softmax gives P, and O = P V).  Two cuBLAS GEMMs per call
  * (batched over the KV heads of all batches; the G = Hq / Hkv query heads sharing a KV head are
  * stacked as the rows of one GEMM) and one softmax kernel of this library, which also writes
- * LSE.  P is rounded to the I/O type before P V, as on the fused tensor-core paths.
+ * LSE.  The weights are fp16 (p * 2^11) for both I/O types, as on the fused tensor-core paths;
+ * for bf16 I/O, V is first converted to fp16 under a power-of-two scale per KV head in an
+ * internal workspace (allocated on `stream` like fav_forward's, kept until
+ * fav_release_workspace) and O is scaled back and rounded to bf16 by one more kernel.
  *
  *  q, k, v, o, lse, B..dtype   as fav_forward; dtype fp16 or bf16 (else FAV_ERR_UNSUPPORTED)
  *  workspace        device buffer of at least fav_nonflash_workspace_size(B, Hq, Nq, Nkv)
@@ -216,8 +226,11 @@ FAV_API const char *fav_status_string(fav_status s);
 
 /*
  * fav_get_last_device_status -- synchronises the device, then reports and clears the status
- * word that kernels set when one of their bounded waits (on an mbarrier) gave up:
- * FAV_OK or FAV_ERR_DEVICE_TIMEOUT.  FAV_ERR_CUDA if the device could not be queried.
+ * word that kernels set: FAV_ERR_DEVICE_TIMEOUT when one of their bounded waits (on an
+ * mbarrier) gave up, FAV_ERR_BAD_PAGE when fav_decode_paged met an out-of-range block-table
+ * entry, FAV_ERR_DEVICE_CHECK when a check of the self-checking build failed; FAV_OK if none
+ * did since the last call (the last one set wins).  FAV_ERR_CUDA if the device could not be
+ * queried.
  */
 FAV_API fav_status fav_get_last_device_status(void);
 
@@ -251,6 +264,18 @@ FAV_API int fav_last_decode_splits(void);
  * small problems.  The results do not depend on the cap.  FAV_ERR_INVALID_ARG for n < 0.
  */
 FAV_API fav_status fav_set_prefill_grid(int n);
+
+/*
+ * fav_check_wait_timeout -- self-test of the kernels' bounded waits (no counterpart in the
+ * paper: it checks this library's failure reporting).  Launches one warp on `stream` that
+ * waits on a shared-memory mbarrier that nothing ever arrives on, with the same wait code as
+ * the kernels but a give-up limit of limit_us microseconds instead of their 2 s.  The wait gives
+ * up, records FAV_ERR_DEVICE_TIMEOUT in the device status word and the kernel returns normally
+ * (no copy or tensor-core operation is in flight, the context stays usable); read the outcome
+ * with fav_get_last_device_status(), which also clears it.  Asynchronous.
+ * FAV_ERR_INVALID_ARG unless 1 <= limit_us <= 1000000; FAV_ERR_CUDA if the launch failed.
+ */
+FAV_API fav_status fav_check_wait_timeout(int limit_us, void *stream);
 
 /*
  * fav_decode_noalloc -- the decode path (split-KV decode kernel + log-sum-exp combine) with no

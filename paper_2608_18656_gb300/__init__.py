@@ -8,7 +8,7 @@ import ctypes
 import os
 
 __all__ = ["forward", "forward_nonflash", "nonflash_workspace_size", "forward_host", "decode_paged", "prefill_varlen", "Strides", "set_path", "last_path", "set_decode_splits",
-           "last_decode_splits", "set_prefill_grid", "device_status", "release_workspace", "library_path",
+           "last_decode_splits", "set_prefill_grid", "device_status", "check_wait_timeout", "release_workspace", "library_path",
            "FavError", "F32", "F16", "BF16", "PATH_AUTO", "PATH_SIMT", "PATH_DECODE",
            "PATH_PREFILL"]
 
@@ -17,10 +17,13 @@ PATH_AUTO, PATH_SIMT, PATH_DECODE, PATH_PREFILL = 0, 1, 2, 3
 PATH_NAMES = {PATH_AUTO: "auto", PATH_SIMT: "simt", PATH_DECODE: "decode",
               PATH_PREFILL: "prefill"}
 STATUS_NAMES = {0: "FAV_OK", 1: "FAV_ERR_INVALID_ARG", 2: "FAV_ERR_UNSUPPORTED",
-                3: "FAV_ERR_CUDA", 4: "FAV_ERR_NO_MEMORY", 5: "FAV_ERR_DEVICE_TIMEOUT"}
+                3: "FAV_ERR_CUDA", 4: "FAV_ERR_NO_MEMORY", 5: "FAV_ERR_DEVICE_TIMEOUT",
+                6: "FAV_ERR_DEVICE_CHECK", 7: "FAV_ERR_BAD_PAGE"}
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_LIB_PATH = os.path.join(_HERE, "libfav.so")
+# FAV_LIBRARY in the environment selects another build of the library (the self-checking
+# -DFAV_DEBUG_CHECKS variant, libfav_debug.so); by default the in-tree libfav.so.
+_LIB_PATH = os.environ.get("FAV_LIBRARY") or os.path.join(_HERE, "libfav.so")
 _lib = None
 
 
@@ -84,6 +87,8 @@ def lib():
         L.fav_last_decode_splits.restype = i
         L.fav_set_prefill_grid.argtypes = [i]
         L.fav_set_prefill_grid.restype = i
+        L.fav_check_wait_timeout.argtypes = [i, vp]
+        L.fav_check_wait_timeout.restype = i
         _lib = L
     return _lib
 
@@ -316,6 +321,15 @@ def set_prefill_grid(n):
 def device_status():
     """Synchronises; returns and clears the kernels' bounded-wait status (0 = ok)."""
     return lib().fav_get_last_device_status()
+
+
+def check_wait_timeout(limit_us=1000, stream=None):
+    """Launches the bounded-wait self-test (fav_check_wait_timeout) on the current torch stream
+    (or `stream`): one warp waits on an mbarrier that nothing arrives on and gives up after
+    limit_us; the outcome is read with device_status()."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    _check(lib().fav_check_wait_timeout(int(limit_us), s.cuda_stream))
 
 
 def release_workspace():

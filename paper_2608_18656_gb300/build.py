@@ -23,8 +23,8 @@ def nvcc():
     return path if os.path.exists(path) else "nvcc"
 
 
-def compile_one(src, extra=()):
-    obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
+def compile_one(src, extra=(), objdir=BUILD):
+    obj = os.path.join(objdir, os.path.splitext(src)[0] + ".o")
     cmd = [nvcc(), *ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
            "-Xcompiler", "-fvisibility=hidden", "-I", os.path.join(HERE, "..", "include"),
            *extra, "-c", os.path.join(CSRC, src), "-o", obj]
@@ -34,21 +34,33 @@ def compile_one(src, extra=()):
     return obj, r.stderr
 
 
-def build(verbose=False, extra=()):
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose=False, extra=(), lib=LIB, objdir=BUILD):
+    """Compiles every translation unit (with the extra nvcc flags) into objdir and links lib."""
+    os.makedirs(objdir, exist_ok=True)
     with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        results = list(ex.map(lambda s: compile_one(s, extra), SOURCES))
+        results = list(ex.map(lambda s: compile_one(s, extra, objdir), SOURCES))
     if verbose:
         for _, log in results:
             if log:
                 sys.stderr.write(log)
-    tmp = LIB + ".tmp.%d" % os.getpid()
+    tmp = lib + ".tmp.%d" % os.getpid()
     cmd = [nvcc(), *ARCH, "-shared", "-cudart", "static", "-ldl", "-o", tmp] + [o for o, _ in results]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError("link failed:\n%s%s" % (r.stdout, r.stderr))
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
+
+
+# The self-checking variant (-DFAV_DEBUG_CHECKS: shared-memory bounds, TMA destination
+# alignment, global indices, per-role unit and tile totals; a violation prints, sets device
+# status 6 and skips the access).  Load it with FAV_LIBRARY=<DEBUG_LIB> in the environment.
+DEBUG_LIB = os.path.join(HERE, "libfav_debug.so")
+DEBUG_BUILD = os.path.join(HERE, "_build_debug")
+
+
+def build_debug(verbose=False):
+    return build(verbose, ("-DFAV_DEBUG_CHECKS",), DEBUG_LIB, DEBUG_BUILD)
 
 
 if __name__ == "__main__":

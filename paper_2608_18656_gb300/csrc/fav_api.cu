@@ -13,17 +13,33 @@
 #include <atomic>
 #include <mutex>
 
+#include "fav_device.cuh"
 #include "fav_internal.h"
 
 // Status word written by kernels whose bounded waits gave up (FAV_ERR_DEVICE_TIMEOUT).
 __device__ int g_fav_device_status;
+
+// Self-test of the bounded waits: one warp initialises a shared-memory mbarrier that nothing
+// arrives on and waits for its first phase with the kernels' own wait (fav::mbar_wait_il),
+// given up after limit_ns instead of FAV_WAIT_NS.  No copy and no tensor-core operation is in
+// flight; the kernel records the give-up in *status and returns.
+__global__ void __launch_bounds__(32) fav_wait_probe_kernel(int *status, unsigned long long limit_ns) {
+    __shared__ unsigned long long bar_word;
+    const uint32_t bar = fav::smem_u32(&bar_word);
+    if (threadIdx.x == 0) {
+        fav::mbar_init(bar, 1);
+        fav::mbar_fence_init();
+    }
+    __syncwarp();
+    (void)__all_sync(~0u, fav::mbar_wait_il(bar, 0, status, limit_ns));
+}
 
 namespace {
 
 constexpr int kMaxDevices = 64;
 
 struct DeviceState {
-    bool init = false;
+    std::atomic<bool> init{false};   // set once, under g_mu, after the fields below
     int *status = nullptr;     // device address of g_fav_device_status
     int num_sms = 0;
     void *ws = nullptr;        // split-KV partials
@@ -49,19 +65,24 @@ std::atomic<int> g_splits{0};
 std::atomic<int> g_last_splits{0};
 std::atomic<int> g_prefill_grid{0};
 
+// The calling thread's current device's state, set up on first use (under g_mu, so that two
+// threads' first calls on one device do not race).  Callers must not hold g_mu.
 fav_status device_state(DeviceState **out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FAV_ERR_CUDA;
     DeviceState &d = g_dev[dev];
-    if (!d.init) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_fav_device_status) != cudaSuccess) return FAV_ERR_CUDA;
-        int sms = 0;
-        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-            return FAV_ERR_CUDA;
-        d.status = static_cast<int *>(p);
-        d.num_sms = sms;
-        d.init = true;
+    if (!d.init.load(std::memory_order_acquire)) {
+        std::lock_guard<std::mutex> lk(g_mu);
+        if (!d.init.load(std::memory_order_relaxed)) {
+            void *p = nullptr;
+            if (cudaGetSymbolAddress(&p, g_fav_device_status) != cudaSuccess) return FAV_ERR_CUDA;
+            int sms = 0;
+            if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+                return FAV_ERR_CUDA;
+            d.status = static_cast<int *>(p);
+            d.num_sms = sms;
+            d.init.store(true, std::memory_order_release);
+        }
     }
     *out = &d;
     return FAV_OK;
@@ -519,11 +540,24 @@ fav_status fav_forward_nonflash(const void *q, const void *k, const void *v, voi
     if (lse && !aligned(lse, 4)) return FAV_ERR_INVALID_ARG;
     fav_status st = validate_shape(B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
     if (st != FAV_OK) return st;
-    const FavArgs a = make_args(q, k, v, o, lse, B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
+    FavArgs a = make_args(q, k, v, o, lse, B, Hq, Hkv, Nq, Nkv, D, scale, causal, dtype);
     if (!fav_nonflash_shape_ok(a)) return FAV_ERR_UNSUPPORTED;
     if (workspace_bytes < fav_nonflash_workspace_bytes(a)) return FAV_ERR_INVALID_ARG;
     if (!fav_nonflash_available()) return FAV_ERR_UNSUPPORTED;
-    return fav_launch_nonflash(a, workspace, static_cast<cudaStream_t>(stream));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    void *vws = nullptr;
+    if (dtype == FAV_BF16) {   // the fp16 copy of V (internal, as for fav_forward's bf16 prefill)
+        DeviceState *ds = nullptr;
+        st = device_state(&ds);
+        if (st != FAV_OK) return st;
+        a.num_sms = ds->num_sms;
+        std::lock_guard<std::mutex> lk(g_mu);
+        st = ensure_buffer(&ds->ws_pre, &ds->ws_pre_bytes, fav_v16_workspace_bytes(a), s);
+        if (st != FAV_OK) return st;
+        vws = ds->ws_pre;
+    }
+    cudaGetLastError();
+    return fav_launch_nonflash(a, workspace, vws, s);
 }
 
 fav_status fav_forward_host(const void *q, const void *k, const void *v, void *o, float *lse,
@@ -617,6 +651,8 @@ const char *fav_status_string(fav_status s) {
     case FAV_ERR_CUDA: return "CUDA runtime error";
     case FAV_ERR_NO_MEMORY: return "workspace allocation failed";
     case FAV_ERR_DEVICE_TIMEOUT: return "a bounded device wait timed out";
+    case FAV_ERR_DEVICE_CHECK: return "a device-side check of the self-checking build failed";
+    case FAV_ERR_BAD_PAGE: return "a block-table entry lies outside the page pool";
     }
     return "unknown status";
 }
@@ -661,6 +697,17 @@ fav_status fav_set_decode_splits(int n) {
 }
 
 int fav_last_decode_splits(void) { return g_last_splits.load(); }
+
+fav_status fav_check_wait_timeout(int limit_us, void *stream) {
+    if (limit_us < 1 || limit_us > 1000000) return FAV_ERR_INVALID_ARG;
+    DeviceState *ds = nullptr;
+    const fav_status st = device_state(&ds);
+    if (st != FAV_OK) return st;
+    cudaGetLastError();
+    fav_wait_probe_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(
+        ds->status, 1000ull * (unsigned long long)limit_us);
+    return cudaGetLastError() == cudaSuccess ? FAV_OK : FAV_ERR_CUDA;
+}
 
 fav_status fav_set_prefill_grid(int n) {
     if (n < 0) return FAV_ERR_INVALID_ARG;

@@ -124,13 +124,24 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         const CUtensorMap *tm = is_v ? &tmV : &tmK;
         if constexpr (kPaged) {
             // page id of box e (tile e / bpt, rows (e % bpt) * box_rows .. + box_rows); boxes
-            // past the sequence read page 0 (their keys are masked).  Filled by the K warp;
-            // both producer warps then meet at a named barrier (neither leaves before it).
+            // past the sequence read page 0 (their keys are masked).  A block-table entry outside
+            // [0, num_pages) sets the device status word (FAV_ERR_BAD_PAGE) and is stored as -1:
+            // the copy reads the zero fill and the consumers mask that box's keys, so they take
+            // no part in the softmax.  Filled by the K warp; both producer warps then meet at a
+            // named barrier (neither leaves before it).
             if (!is_v) {
                 const int n_box = my_tiles * bpt;
                 for (int e = lane; e < n_box && e < Cfg::kPageSlots; e += 32) {
                     const int key = (tile0 + e / bpt) * TK + (e % bpt) * box_rows;
-                    page_list[e] = key < Nkv ? pg.block_table[(long long)b * pg.max_pages + key / pg.page_size] : 0;
+                    int pid = 0;
+                    if (key < Nkv) {
+                        pid = pg.block_table[(long long)b * pg.max_pages + key / pg.page_size];
+                        if (pid < 0 || pid >= pg.num_pages) {
+                            atomicExch(status, (int)FAV_ERR_BAD_PAGE);
+                            pid = -1;
+                        }
+                    }
+                    page_list[e] = pid;
                 }
             }
             fav::named_bar_sync(2, 64);
@@ -242,8 +253,15 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
             }
         }
 
-        // Mask, scale into the log2 domain, online softmax.
-        const bool need_mask = key0 + TK > lim_min;
+        // Mask, scale into the log2 domain, online softmax.  (Paged: boxes whose block-table
+        // entry was out of range, bad_boxes bit i for rows i * box_rows .. of the tile, are
+        // masked as well.)
+        uint32_t bad_boxes = 0;
+        if constexpr (kPaged) {
+            for (int i = 0; i < bpt; ++i)
+                if (page_list[lt * bpt + i] < 0) bad_boxes |= 1u << i;
+        }
+        const bool need_mask = key0 + TK > lim_min || bad_boxes != 0;
         float mx[2] = {-INFINITY, -INFINITY};
 #pragma unroll
         for (int nt = 0; nt < TK / 8; ++nt) {
@@ -253,6 +271,7 @@ fav_decode_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
                 if (need_mask) {
                     const int j = key0 + 8 * nt + 2 * t + (e & 1);
                     if (j >= lim[e >> 1]) x = -INFINITY;
+                    if (kPaged && ((bad_boxes >> ((j - key0) / box_rows)) & 1u)) x = -INFINITY;
                 }
                 s[nt][e] = x;
                 mx[e >> 1] = fmaxf(mx[e >> 1], x);

@@ -7,6 +7,8 @@
 #include <stdint.h>
 #include <stdio.h>
 
+#include "../../include/fav.h"
+
 #ifndef FAV_WAIT_NS
 #define FAV_WAIT_NS 2000000000ull   // a wait that lasts 2 s is a hang: give up, flag it
 #endif
@@ -23,7 +25,7 @@ static __device__ int g_fav_check_prints;
                     ? printf("[fav check] %s:%d block (%d,%d,%d) thread %d: %s\n", __FILE__,   \
                              __LINE__, blockIdx.x, blockIdx.y, blockIdx.z, threadIdx.x, #cond) \
                     : 0),                                                                      \
-               atomicExch((status), 6), false))
+               atomicExch((status), (int)FAV_ERR_DEVICE_CHECK), false))
 #else
 #define FAV_CHECK(cond, status) true
 #endif
@@ -141,13 +143,15 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int *st
 
 // The same bounded waits with the slow path inlined, for kernels whose warp roles run under
 // setmaxnreg register budgets (a call to an out-of-line function cannot be register-allocated
-// inside such a role).
-__device__ __forceinline__ bool mbar_wait_il(uint32_t bar, uint32_t parity, int *status) {
+// inside such a role).  limit_ns: the give-up time (the kernels use FAV_WAIT_NS; the wait
+// self-test of fav_check_wait_timeout passes a short one).
+__device__ __forceinline__ bool mbar_wait_il(uint32_t bar, uint32_t parity, int *status,
+                                             uint64_t limit_ns = FAV_WAIT_NS) {
     if (mbar_try(bar, parity)) return true;
     const uint64_t t0 = globaltimer();
     while (true) {
         if (mbar_try(bar, parity)) return true;
-        if (globaltimer() - t0 > FAV_WAIT_NS) {
+        if (globaltimer() - t0 > limit_ns) {
             atomicExch(status, 5);
             return false;
         }

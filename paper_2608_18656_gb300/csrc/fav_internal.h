@@ -77,13 +77,16 @@ fav_status fav_launch_prefill_pair_varlen(const FavArgs &a, const int4 *units, i
 fav_status fav_launch_prefill(const FavArgs &a, void *workspace, cudaStream_t s);
 
 // Non-fused attention (fav_nonflash.cu): cuBLAS S = scale Q K^T (fp32), masked row softmax
-// (weights in place over S, LSE), cuBLAS O = P V.  workspace: fav_nonflash_workspace_bytes.
+// (fp16 weights * 2^11 in place over S, LSE), cuBLAS O = P V.  workspace:
+// fav_nonflash_workspace_bytes; v_workspace (bf16 only): fav_v16_workspace_bytes, for the fp16
+// copy of V and its per-head scales (a.num_sms sizes the conversion grid).
 size_t fav_nonflash_workspace_bytes(const FavArgs &a);
 // Shape limits of this path (fp16/bf16, a score row in shared memory, int GEMM sizes).
 bool fav_nonflash_shape_ok(const FavArgs &a);
 // Whether cuBLAS could be loaded.
 bool fav_nonflash_available();
-fav_status fav_launch_nonflash(const FavArgs &a, void *workspace, cudaStream_t s);
+fav_status fav_launch_nonflash(const FavArgs &a, void *workspace, void *v_workspace,
+                               cudaStream_t s);
 
 // With FAV_DEBUG_SYNC=1 in the environment: synchronise `s` after a launch and report a
 // failure of kernel `what` on stderr.  Returns true if the kernel failed.  No-op otherwise.

@@ -4,10 +4,16 @@
 //   S = scale * Q K^T      one batched GEMM per KV head (its G query heads stacked as the rows),
 //                          fp32 scores in a workspace [B * Hq, Nq, Nkv]
 //   P = softmax(S) (mask)  one block per query row, the row in registers (float4 loads; rows up
-//                          to 8192 keys, a multiple of 4) or else in shared memory; the weights
-//                          (rounded to the I/O type) overwrite the first half of their own fp32
+//                          to 8192 keys, a multiple of 4) or else in shared memory; the weights,
+//                          stored as p * 2^11 in fp16, overwrite the first half of their own fp32
 //                          row, and LSE = max + log(sum)
-//   O = P V                a second batched GEMM per KV head
+//   O = P V                a second batched GEMM per KV head, fp16 x fp16 with alpha = 2^-11
+//
+// The weights are fp16 for both I/O types, as in the fused kernels: 11 significant bits (a bf16
+// weight has 8, and its rounding alone can move O by 2^-9 max|v|), scaled by 2^11 so that weights
+// down to 2^-25 stay fp16 normals.  For bf16 I/O, V is first converted to fp16 under a power of
+// two per KV head (fav_v16_convert, the fused path's conversion), the P V GEMM writes O * 2^-e in
+// fp16 into the output buffer, and fav_nonflash_unscale_kernel turns it into bf16 O in place.
 //
 // The GEMMs are cuBLAS (cublasGemmStridedBatchedEx, fp32 accumulation), loaded on first use with
 // dlopen so that libfav itself does not depend on cuBLAS; without it the entry point returns
@@ -70,7 +76,9 @@ Cublas &cublas() {
 // (bottom-right: key j visible while j <= Nkv - Nq + i), maximum, sum of exponentials, then the
 // weights p_j = exp(s_j - max) / sum rounded to T over the first half of the row's bytes
 // (row stride in T elements: 2 * Nkv), and LSE = max + log(sum).
-template <typename T>
+constexpr float kPScale = 2048.f;       // weights stored as p * 2^11 (fp16)
+constexpr float kPUnscale = 1.f / 2048.f;
+
 __global__ void __launch_bounds__(256)
 fav_nonflash_softmax_kernel(float *__restrict__ s, float *__restrict__ lse, int Nq, int Nkv,
                             int causal) {
@@ -103,16 +111,16 @@ fav_nonflash_softmax_kernel(float *__restrict__ s, float *__restrict__ lse, int 
     __syncthreads();
     sum = 0.f;
     for (int w = 0; w < (int)(blockDim.x >> 5); ++w) sum += red[w];
-    const float inv = sum > 0.f ? 1.f / sum : 0.f;
-    T *p = reinterpret_cast<T *>(src);          // every score of the row is in shared memory
-    for (int j = threadIdx.x; j < Nkv; j += blockDim.x) p[j] = fav::Elem<T>::from_f(row[j] * inv);
+    const float inv = sum > 0.f ? kPScale / sum : 0.f;
+    __half *p = reinterpret_cast<__half *>(src);          // every score of the row is in shared memory
+    for (int j = threadIdx.x; j < Nkv; j += blockDim.x) p[j] = __float2half_rn(row[j] * inv);
     if (lse && threadIdx.x == 0) lse[r] = sum > 0.f ? mx + logf(sum) : -INFINITY;
 }
 
 // The same row softmax with the row in registers, for Nkv % 4 == 0 and Nkv <= 1024 * kVec:
 // each of the 256 threads holds kVec float4 of the row (16-byte loads; causal rows read only
 // their visible prefix), so the row is read once from HBM and the weights written once.
-template <typename T, int kVec>
+template <int kVec>
 __global__ void __launch_bounds__(256)
 fav_nonflash_softmax_reg_kernel(float *__restrict__ s, float *__restrict__ lse, int Nq,
                                 int Nkv, int causal) {
@@ -158,43 +166,62 @@ fav_nonflash_softmax_reg_kernel(float *__restrict__ s, float *__restrict__ lse, 
     sum = 0.f;
 #pragma unroll
     for (int w = 0; w < 8; ++w) sum += red[1][w];
-    const float inv = 1.f / sum;
-    T *p = reinterpret_cast<T *>(src);
+    const float inv = kPScale / sum;
+    __half *p = reinterpret_cast<__half *>(src);
 #pragma unroll
     for (int v = 0; v < kVec; ++v) {
         const int j = 4 * (v * 256 + (int)threadIdx.x);
         if (j < Nkv) {
-            struct alignas(8) T4 { T a, b, c, d; } q;
-            q.a = fav::Elem<T>::from_f(x[v].x * inv);
-            q.b = fav::Elem<T>::from_f(x[v].y * inv);
-            q.c = fav::Elem<T>::from_f(x[v].z * inv);
-            q.d = fav::Elem<T>::from_f(x[v].w * inv);
-            *reinterpret_cast<T4 *>(p + j) = q;
+            const uint2 q = make_uint2(fav::Elem<__half>::pack(x[v].x * inv, x[v].y * inv),
+                                       fav::Elem<__half>::pack(x[v].z * inv, x[v].w * inv));
+            *reinterpret_cast<uint2 *>(p + j) = q;
         }
     }
     if (lse && threadIdx.x == 0) lse[r] = mx + logf(sum);
 }
 
-// The softmax launch for I/O type T: registers when the row fits (and is 16-byte aligned),
-// shared memory otherwise.
-template <typename T>
+// O (fp16, holding O * 2^-e of its KV head: the P V GEMM of the bf16 path) -> bf16 O in place.
+// One thread per 8 elements (16 bytes); rows of D elements, row r = (b * Hq + h) * Nq + i.
+__global__ void __launch_bounds__(256)
+fav_nonflash_unscale_kernel(uint4 *__restrict__ o, const float *__restrict__ v_scale,
+                            long long n8, int D, int Nq, int Hq, int G, int Hkv) {
+    const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+    if (i >= n8) return;
+    const long long r = i * 8 / D;
+    const long long bh = r / Nq;
+    const int h = (int)(bh % Hq);
+    const long long b = bh / Hq;
+    const float sc = v_scale[b * Hkv + h / G];
+    uint4 w = o[i];
+    uint32_t *u = reinterpret_cast<uint32_t *>(&w);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const __half2 x = *reinterpret_cast<const __half2 *>(&u[k]);
+        const float2 f = __half22float2(x);
+        u[k] = fav::Elem<__nv_bfloat16>::pack(f.x * sc, f.y * sc);
+    }
+    o[i] = w;
+}
+
+// The softmax launch: registers when the row fits (and is 16-byte aligned), shared memory
+// otherwise.
 cudaError_t launch_softmax(float *S, float *lse, long long rows, int Nq, int Nk, int causal,
                            cudaStream_t stream) {
     const unsigned grid = (unsigned)rows;
     if (Nk % 4 == 0 && Nk <= 8192) {
         const int vec = (Nk + 1023) / 1024;
         if (vec <= 1)
-            fav_nonflash_softmax_reg_kernel<T, 1><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
+            fav_nonflash_softmax_reg_kernel<1><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
         else if (vec <= 2)
-            fav_nonflash_softmax_reg_kernel<T, 2><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
+            fav_nonflash_softmax_reg_kernel<2><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
         else if (vec <= 4)
-            fav_nonflash_softmax_reg_kernel<T, 4><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
+            fav_nonflash_softmax_reg_kernel<4><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
         else
-            fav_nonflash_softmax_reg_kernel<T, 8><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
+            fav_nonflash_softmax_reg_kernel<8><<<grid, 256, 0, stream>>>(S, lse, Nq, Nk, causal);
         return cudaGetLastError();
     }
     const size_t smem = (size_t)Nk * sizeof(float);
-    auto kern = fav_nonflash_softmax_kernel<T>;
+    auto kern = fav_nonflash_softmax_kernel;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)(smem > 48 * 1024 ? smem : 48 * 1024));
     if (e != cudaSuccess) return e;
@@ -217,7 +244,8 @@ bool fav_nonflash_shape_ok(const FavArgs &a) {
 
 bool fav_nonflash_available() { return cublas().ok; }
 
-fav_status fav_launch_nonflash(const FavArgs &a, void *workspace, cudaStream_t stream) {
+fav_status fav_launch_nonflash(const FavArgs &a, void *workspace, void *v_workspace,
+                               cudaStream_t stream) {
     Cublas &c = cublas();
     if (!c.ok) return FAV_ERR_UNSUPPORTED;
     int dev = 0;
@@ -229,24 +257,40 @@ fav_status fav_launch_nonflash(const FavArgs &a, void *workspace, cudaStream_t s
     if (c.set_stream(c.handle[dev], stream) != 0) return FAV_ERR_CUDA;
     const int G = a.Hq / a.Hkv, N = a.Nq, Nk = a.Nkv, D = a.D, M = G * N;
     const int batch = a.B * a.Hkv;
-    const int io = a.dtype == FAV_F16 ? kCudaR16F : kCudaR16BF;
+    const bool bf = a.dtype == FAV_BF16;
+    const int io = bf ? kCudaR16BF : kCudaR16F;
     float *S = static_cast<float *>(workspace);
-    const float alpha_s = a.scale, one = 1.f, zero = 0.f;
+    const float alpha_s = a.scale, alpha_o = kPUnscale, zero = 0.f;
+    // bf16: V as fp16 under a power of two per KV head (contiguous [B, Hkv, Nkv, D])
+    const void *v16 = a.v;
+    const float *v_scale = nullptr;
+    if (bf) {
+        FavStrides vs16;
+        const fav_status st = fav_v16_convert(a, v_workspace, stream, &v16, &vs16, &v_scale);
+        if (st != FAV_OK) return st;
+    }
     // S^T (Nk x M, column-major) = K (Nk x D) . Q^T (D x M): row-major S = Q K^T, per KV head
     if (c.gemm(c.handle[dev], kCublasOpT, kCublasOpN, Nk, M, D, &alpha_s, a.k, io, D,
                (long long)Nk * D, a.q, io, D, (long long)M * D, &zero, S, kCudaR32F, Nk,
                (long long)M * Nk, batch, kCublasCompute32F, kCublasGemmDefault) != 0)
         return FAV_ERR_CUDA;
     const long long rows = (long long)a.B * a.Hq * N;
-    const cudaError_t e = a.dtype == FAV_F16
-                              ? launch_softmax<__half>(S, a.lse, rows, N, Nk, a.causal, stream)
-                              : launch_softmax<__nv_bfloat16>(S, a.lse, rows, N, Nk, a.causal, stream);
+    const cudaError_t e = launch_softmax(S, a.lse, rows, N, Nk, a.causal, stream);
     if (e != cudaSuccess || fav_debug_sync("fav_nonflash_softmax_kernel", stream))
         return FAV_ERR_CUDA;
-    // O^T (D x M) = V^T (D x Nk) . P^T (Nk x M); P rows are 2 * Nk elements apart (in place)
-    if (c.gemm(c.handle[dev], kCublasOpN, kCublasOpN, D, M, Nk, &one, a.v, io, D,
-               (long long)Nk * D, S, io, 2 * Nk, (long long)M * Nk * 2, &zero, a.o, io, D,
-               (long long)M * D, batch, kCublasCompute32F, kCublasGemmDefault) != 0)
+    // O^T (D x M) = 2^-11 V^T (D x Nk) . P^T (Nk x M), all fp16; P rows are 2 * Nk elements
+    // apart (in place).  fp16 I/O: O itself; bf16 I/O: O * 2^-e, converted in place below.
+    if (c.gemm(c.handle[dev], kCublasOpN, kCublasOpN, D, M, Nk, &alpha_o, v16, kCudaR16F, D,
+               (long long)Nk * D, S, kCudaR16F, 2 * Nk, (long long)M * Nk * 2, &zero, a.o,
+               kCudaR16F, D, (long long)M * D, batch, kCublasCompute32F, kCublasGemmDefault) != 0)
         return FAV_ERR_CUDA;
+    if (bf) {
+        const long long n8 = rows * D / 8;
+        fav_nonflash_unscale_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, stream>>>(
+            static_cast<uint4 *>(a.o), v_scale, n8, D, N, a.Hq, G, a.Hkv);
+        if (cudaGetLastError() != cudaSuccess ||
+            fav_debug_sync("fav_nonflash_unscale_kernel", stream))
+            return FAV_ERR_CUDA;
+    }
     return FAV_OK;
 }

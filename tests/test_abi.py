@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol():
 
 def test_status_strings():
     L = fav.lib()
-    for code in range(6):
+    for code in range(8):
         assert L.fav_status_string(code)
     assert L.fav_status_string(99) == b"unknown status"
 
@@ -99,3 +99,8 @@ def test_python_binding_has_no_cpu_path():
     q = torch.zeros(1, 1, 4, 64, dtype=torch.float16)
     with pytest.raises(ValueError):
         fav.forward(q, q, q)
+
+
+@pytest.mark.parametrize("limit_us", [0, -1, 1000001])
+def test_wait_self_test_rejects_limits(limit_us):
+    assert fav.lib().fav_check_wait_timeout(limit_us, None) == 1   # FAV_ERR_INVALID_ARG

@@ -1,30 +1,18 @@
 """fav_forward_nonflash (materialised scores, cuBLAS GEMMs + this library's softmax kernel)
-against the fp64 oracle on seeded inputs (needs a GB300)."""
+against the fp64 oracle on seeded inputs (needs a GB300), with the library's tolerances (O
+within 3e-3 for fp16 and bf16, LSE within 1e-4)."""
 import numpy as np
 import pytest
 
 import paper_2608_18656_gb300 as fav
 from paper_2608_18656_gb300 import inputs as I
-import gpu_util
-from gpu_util import check, sample_rows, to_device
+from gpu_util import check, to_device
 
 pytestmark = pytest.mark.gpu
 
 
 def W(dtype, B, Hq, Hkv, Nq, Nkv, D, causal=False, outliers=False, seed=7):
     return I.Workload("t", dtype, B, Hq, Hkv, Nq, Nkv, D, causal, outliers, seed)
-
-
-# Tolerance on O.  fp16: the library's 3e-3.  bf16: this path rounds the normalised weights P
-# to bf16 (8 significant bits, unit roundoff u = 2^-8) before P V, where the fused kernels use
-# fp16 weights; so |sum_j p_j d_j v_j| <= u max|v| with sum_j p_j = 1, plus the final rounding
-# of O to bf16, u |O| <= u max|v|: 2 * 2^-8 * max|v|, and every input here has |v| <= 1.
-NONFLASH_O_TOL = {I.F16: gpu_util.O_TOL[I.F16], I.BF16: 2.0 ** -7}
-
-
-@pytest.fixture(autouse=True)
-def _nonflash_tolerance(monkeypatch):
-    monkeypatch.setattr(gpu_util, "O_TOL", {**gpu_util.O_TOL, **NONFLASH_O_TOL})
 
 
 def run_nonflash(w, x, workspace=None):
@@ -67,9 +55,9 @@ def test_nonflash_outliers_and_caller_workspace():
 
 
 @pytest.mark.parametrize("idx", [1, 2])
-def test_nonflash_prefill_workloads_sampled(idx):
-    """The measured prefill workloads at full size, on sampled rows."""
+def test_nonflash_prefill_workloads(idx):
+    """The measured prefill workloads at full size, every row."""
     w = I.WORKLOADS[idx]
     x = I.make_inputs(w)
     o, lse = run_nonflash(w, x)
-    check(w, o, lse, x, rows=sample_rows(w, 2048, seed=idx))
+    check(w, o, lse, x)

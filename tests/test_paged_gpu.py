@@ -140,3 +140,34 @@ def test_paged_equals_dense_decode_bitwise():
     torch.cuda.synchronize()
     np.testing.assert_array_equal(o, od.float().cpu().numpy().astype(np.float64))
     np.testing.assert_array_equal(lse, ld.cpu().numpy().astype(np.float64))
+
+
+@pytest.mark.parametrize("splits", [0, 3])
+def test_out_of_range_page_ids_are_reported_and_left_out(splits):
+    """Block-table entries outside [0, num_pages) inside a sequence's length: the call reports
+    FAV_ERR_BAD_PAGE through the device status word, and the keys of those pages take no part in
+    the softmax (every other key is attended as usual)."""
+    import torch
+    fav.set_decode_splits(splits)
+    dtype, D, Hq, Hkv, page = I.BF16, 128, 8, 2, 16
+    lens = [100, 70]
+    x = build(dtype, lens, Hq, Hkv, 1, D, page, seed=9)
+    x["table"][0, 2] = x["num_pages"] + 5      # keys 32..47 of sequence 0
+    x["table"][1, 0] = -3                      # keys 0..15 of sequence 1
+    scale = float(np.float32(1.0 / np.sqrt(D)))
+    q = to_device(I.to_storage(x["q"], dtype), dtype)
+    kc = to_device(I.to_storage(x["pool_k"], dtype), dtype)
+    vc = to_device(I.to_storage(x["pool_v"], dtype), dtype)
+    o, lse = fav.decode_paged(q, kc, vc, torch.from_numpy(x["table"]).cuda(),
+                              torch.from_numpy(x["lens"]).cuda(), causal=False, scale=scale)
+    torch.cuda.synchronize()
+    assert fav.device_status() == 7                     # FAV_ERR_BAD_PAGE
+    assert fav.device_status() == 0
+    o = o.float().cpu().numpy().astype(np.float64)
+    lse = lse.cpu().numpy().astype(np.float64)
+    for b, dropped in ((0, range(32, 48)), (1, range(0, 16))):
+        k, v = x["dense"][b]
+        keep = np.array([j for j in range(k.shape[2]) if j not in dropped])
+        ro, rl = oracle.attention(x["q"][b:b + 1], k[:, :, keep], v[:, :, keep], scale, False)
+        assert np.abs(o[b] - ro[0]).max() <= O_TOL[dtype]
+        assert np.abs(lse[b] - rl[0]).max() <= LSE_TOL
