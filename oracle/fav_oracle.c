@@ -15,7 +15,7 @@
  *   O    = sum_j exp(s_j - m) * V[b,g,j,:] / l
  *   LSE  = m + ln l
  *
- * Readings of points the paper leaves open (each one is also listed in the design doc):
+ * Readings of points the paper leaves open:
  *  - g = h / (Hq / Hkv): consecutive query heads share one K/V head (Method section on GQA,
  *    where one loaded K row is replicated over the adjacent head slots of a register).
  *  - causal masking (Algorithm "ggml-vec FlashAttention" and Algorithm "FlashAttention-V for
