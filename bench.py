@@ -33,7 +33,8 @@ from paper_2608_18656_gb300 import inputs as I  # noqa: E402
 
 HEADLINE = 1          # index of the headline workload in inputs.WORKLOADS
 METRIC = "attention TFLOP/s (prefill) and KV GB/s (decode) on 1 GB300, % of roofline"
-EXTRA = [2, 3, 4]     # reported alongside
+EXTRA = [0, 2, 3, 4]  # reported alongside (0: the exact fp32 path, timed without a roofline claim)
+VARLEN = 0            # index in inputs.VARLEN_WORKLOADS of the packed-batch workload (extra)
 
 
 def parse():
@@ -45,6 +46,7 @@ def parse():
     ap.add_argument("--no-extra", action="store_true", help="headline workload only")
     ap.add_argument("--extra", default=None,
                     help="comma-separated indices of the extra workloads to time (default: all)")
+    ap.add_argument("--no-varlen", action="store_true", help="skip the packed-batch workload")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle cpu_baseline")
     ap.add_argument("--no-nonflash", action="store_true",
                     help="skip the non-fused comparison (materialised scores) on the headline")
@@ -347,14 +349,25 @@ def fav_arm(args, dist):
                                "roofline": {"bound": "hbm", "achieved": gbs / dist.world,
                                             "peak": pk["hbm_gbs"], "unit": "GB/s",
                                             "frac": gbs / dist.world / pk["hbm_gbs"],
-                                            "frac_of_nominal_7900": gbs / dist.world / 7900.0}})
+                                            "frac_of_nominal_7900": gbs / dist.world / 7900.0,
+                                            "traffic": traffic_of(we)}})
+            elif we.dtype == I.F32:
+                tf = job_rate(we.flops, mse * 1e-3, dist.world) / 1e12
+                extras.append({"workload": we.name, "value": tf, "unit": "TFLOP/s",
+                               "us_per_step": mse * 1e3, "ms_per_step": mse, "path": pe,
+                               "kernel_launches_per_step": nle, "roofline": None,
+                               "note": "exact fp32 CUDA-core path on 8.4 MFLOP: launch-latency "
+                                       "bound, reported without a roofline claim"})
             else:
                 tf = job_rate(we.flops, mse * 1e-3, dist.world) / 1e12
                 extras.append({"workload": we.name, "value": tf, "unit": "TFLOP/s",
                                "ms_per_step": mse, "path": pe, "kernel_launches_per_step": nle,
                                "roofline": {"bound": "tensor", "achieved": tf / dist.world,
                                             "peak": pk["tflops"], "unit": "TFLOP/s",
-                                            "frac": tf / dist.world / pk["tflops"]}})
+                                            "frac": tf / dist.world / pk["tflops"],
+                                            "traffic": traffic_of(we)}})
+    if not args.no_extra and not args.no_varlen:
+        extras.append(bench_varlen(fav, I.VARLEN_WORKLOADS[VARLEN], args, stream, dist, pk))
     nonflash = None
     if not args.no_nonflash:
         nonflash = bench_nonflash(fav, w, x, args, stream, dist, ms)
@@ -375,12 +388,7 @@ def fav_arm(args, dist):
         cpu = {"value": flops / t / 1e12, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
                "sample": "%d of %d query rows of %s, fp64, %.2f s"
                          % (len(rows), w.B * w.Hq * w.Nq, w.name, t)}
-    traffic = None
-    tpath = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tpath):
-        tr = json.load(open(tpath)).get(w.name)
-        if tr and tr.get("kernel_source_hash") == kernel_hash():
-            traffic = tr.get("dram_bytes_per_launch")
+    traffic = traffic_of(w)
     line = {
         "metric": METRIC,
         "value": value, "unit": "TFLOP/s", "n_gpus": dist.world, "steps": args.steps,
@@ -435,20 +443,75 @@ def bench_nonflash(fav, w, x, args, stream, dist, fused_ms):
                        "cuBLAS O = P V"}
 
 
-def kernel_hash():
-    """Hash of the code (comments and whitespace removed) of the sources the headline (prefill,
-    D = 128) kernel is compiled from: the traffic figure recorded under profiles/ is used only
-    while that code is unchanged."""
+def bench_varlen(fav, w, args, stream, dist, pk):
+    """The packed batch of short prompts through fav_prefill_varlen (one call per step: the
+    host builds the unit list and copies it to the device, then one launch of the prefill
+    kernel)."""
+    import torch
+    x = I.make_varlen_inputs(w)
+    dev = {n: torch.from_numpy(x[n + "_bits"]).cuda() for n in ("q", "k", "v")}
+    cu = x["cu_seqlens"]
+    o = torch.empty_like(dev["q"])
+    lse = torch.empty((w.Hq, int(cu[-1])), dtype=torch.float32, device="cuda")
+
+    def step():
+        fav.prefill_varlen(dev["q"], dev["k"], dev["v"], cu, cu, causal=w.causal, scale=w.scale,
+                           out=o, lse_out=lse, stream=stream)
+    step()
+    torch.cuda.synchronize()
+    if fav.device_status() != 0:
+        raise RuntimeError("device wait timed out in %s" % w.name)
+    times, _ = time_device(step, args.steps, args.warmup, stream, dist)
+    ms = dist.max(statistics.mean(times))
+    tf = job_rate(w.flops, ms * 1e-3, dist.world) / 1e12
+    return {"workload": w.name, "value": tf, "unit": "TFLOP/s", "ms_per_step": ms,
+            "path": "prefill (packed batch)", "kernel_launches_per_step": 1,
+            "sequences": w.n_seq, "tokens": int(cu[-1]),
+            "roofline": {"bound": "tensor", "achieved": tf / dist.world, "peak": pk["tflops"],
+                         "unit": "TFLOP/s", "frac": tf / dist.world / pk["tflops"],
+                         "traffic": traffic_of(w)}}
+
+
+# Sources each workload's dominant kernel is compiled from (for the traffic record's hash).
+KERNEL_SOURCES = {
+    "prefill_d128": ("fav_prefill.cu", "fav_device.cuh", "fav_tc.cuh"),
+    "prefill_d64": ("fav_prefill_pair.cu", "fav_device.cuh", "fav_tc.cuh"),
+    "decode": ("fav_decode.cu", "fav_device.cuh"),
+}
+
+
+def kernel_family(w):
+    if getattr(w, "Nq", 0) == 1:
+        return "decode"
+    return "prefill_d128" if w.D == 128 else "prefill_d64"
+
+
+def kernel_hash(family="prefill_d128"):
+    """Hash of the code (comments and whitespace removed) of the sources a workload's dominant
+    kernel is compiled from: a traffic figure recorded under profiles/ is used only while that
+    code is unchanged."""
     import hashlib
     import re
     h = hashlib.sha256()
     src = os.path.join(ROOT, "paper_2608_18656_gb300", "csrc")
-    for f in ("fav_prefill.cu", "fav_device.cuh", "fav_tc.cuh"):
+    for f in KERNEL_SOURCES[family]:
         text = open(os.path.join(src, f)).read()
         text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)      # block comments
         text = re.sub(r"//[^\n]*", " ", text)                    # line comments
         h.update(" ".join(text.split()).encode())
     return h.hexdigest()[:16]
+
+
+def traffic_of(w):
+    """DRAM bytes (read + write) of one launch of the workload's dominant kernel, from the ncu
+    record in profiles/traffic.json, or None if there is none for the current kernel code."""
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(tpath):
+        return None
+    tr = json.load(open(tpath)).get(w.name)
+    if tr and tr.get("kernel_source_hash") == kernel_hash(kernel_family(w)):
+        return tr.get("dram_bytes_per_launch")
+    return None
 
 
 def main():

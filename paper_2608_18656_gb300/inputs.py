@@ -85,6 +85,67 @@ WORKLOADS = [
 ]
 
 
+@dataclass(frozen=True)
+class VarlenWorkload:
+    """A packed batch of prompts of different lengths (the paper's short edge prompts, N from 64
+    to 512 tokens): n_seq lengths drawn uniformly from [lo, hi] (seeded), each sequence attending
+    to itself; Q [total, Hq, D], K and V [total, Hkv, D] (token-major, cu_seqlens layout)."""
+    name: str
+    dtype: int
+    n_seq: int
+    lo: int
+    hi: int
+    Hq: int
+    Hkv: int
+    D: int
+    causal: bool
+    seed: int
+
+    @property
+    def scale(self):
+        return float(np.float32(1.0 / np.sqrt(self.D)))
+
+    @property
+    def lengths(self):
+        rng = np.random.Generator(np.random.PCG64(self.seed))
+        return rng.integers(self.lo, self.hi + 1, size=self.n_seq)
+
+    @property
+    def cu_seqlens(self):
+        return np.concatenate([[0], np.cumsum(self.lengths)]).astype(np.int32)
+
+    @property
+    def flops(self):
+        """Algorithmic FLOPs: 4 * Hq * D per unmasked (query, key) pair of every sequence."""
+        n = self.lengths.astype(np.int64)
+        pairs = n * (n + 1) // 2 if self.causal else n * n
+        return int(4 * self.Hq * self.D * pairs.sum())
+
+
+# Packed-batch workload of the measurement plan: 64 prompts of 64..512 tokens, GQA, fp16.
+VARLEN_WORKLOADS = [
+    VarlenWorkload("varlen_f16_causal_64prompts_n64to512_hq32_hkv8_d128", F16, 64, 64, 512, 32,
+                   8, 128, True, 1240),
+]
+
+
+def make_varlen_inputs(w):
+    """Draw a packed batch: the lengths first (VarlenWorkload.lengths), then Q, K, V as in
+    make_inputs, each [total, H, D]."""
+    rng = np.random.Generator(np.random.PCG64(w.seed))
+    n = rng.integers(w.lo, w.hi + 1, size=w.n_seq)
+    total = int(n.sum())
+    q = rng.standard_normal((total, w.Hq, w.D))
+    k = rng.standard_normal((total, w.Hkv, w.D))
+    v = rng.uniform(-1.0, 1.0, (total, w.Hkv, w.D))
+    out = {"cu_seqlens": np.concatenate([[0], np.cumsum(n)]).astype(np.int32)}
+    for name, x in (("q", q), ("k", k), ("v", v)):
+        r = round_to_dtype(x, w.dtype)
+        out[name] = r
+        out[name + "_bits"] = to_storage(r, w.dtype)
+    return out
+
+
 def round_to_dtype(x, dtype):
     """Round fp64 values once, to nearest-even, to the I/O dtype; returns fp64 values."""
     x = np.asarray(x, dtype=np.float64)

@@ -54,3 +54,19 @@ def test_workload_flop_counts():
     assert abs(w.flops / 1e9 - 34.38) < 0.01
     assert abs(I.WORKLOADS[2].flops / 1e9 - 274.9) < 0.1
     assert I.WORKLOADS[3].replace().flops == 4 * 8 * 32 * 128 * 8192
+
+
+def test_varlen_workload_recipe():
+    """The packed-batch workload: lengths in [lo, hi] from the seed (drawn before Q, K, V),
+    offsets consistent with them, inputs of the packed shapes, and the FLOP count of causal
+    self-attention summed over the sequences."""
+    import numpy as np
+    w = I.VARLEN_WORKLOADS[0]
+    n = w.lengths
+    assert len(n) == w.n_seq and n.min() >= w.lo and n.max() <= w.hi
+    x = I.make_varlen_inputs(w)
+    cu = x["cu_seqlens"]
+    assert (cu == w.cu_seqlens).all() and cu[0] == 0 and (np.diff(cu) == n).all()
+    assert x["q"].shape == (cu[-1], w.Hq, w.D) and x["k"].shape == (cu[-1], w.Hkv, w.D)
+    assert w.flops == sum(4 * w.Hq * w.D * int(m) * (int(m) + 1) // 2 for m in n)
+    assert (np.abs(x["v"]) <= 1.0).all()

@@ -131,7 +131,8 @@ def test_decode_outliers():
 @pytest.mark.parametrize("dtype", [I.F32, I.F16, I.BF16])
 @pytest.mark.parametrize("shape", [(1, 2, 2, 1, 1, 64, False), (2, 4, 2, 37, 37, 32, True),
                                    (1, 3, 1, 5, 200, 8, True), (1, 2, 2, 128, 128, 256, False),
-                                   (1, 1, 1, 33, 70, 96, False)])
+                                   (1, 1, 1, 33, 70, 96, False), (1, 2, 1, 6, 300, 4, True),
+                                   (3, 4, 2, 130, 130, 64, True)])
 def test_simt_path(dtype, shape):
     fav.set_path(fav.PATH_SIMT)
     B, Hq, Hkv, Nq, Nkv, D, causal = shape
