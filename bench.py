@@ -45,7 +45,8 @@ def parse():
     ap.add_argument("--impl", default="fav", choices=["fav", "reference"])
     ap.add_argument("--no-extra", action="store_true", help="headline workload only")
     ap.add_argument("--extra", default=None,
-                    help="comma-separated indices of the extra workloads to time (default: all)")
+                    help="comma-separated indices of the extra workloads to time (default: all;"
+                         " an empty string: none of them, the packed batch still runs)")
     ap.add_argument("--no-varlen", action="store_true", help="skip the packed-batch workload")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle cpu_baseline")
     ap.add_argument("--no-nonflash", action="store_true",
@@ -338,7 +339,7 @@ def fav_arm(args, dist):
     x, ms, times, nl, path = bench_workload(w, args.steps, args.warmup)
     extras = []
     if not args.no_extra:
-        chosen = EXTRA if args.extra is None else [int(i) for i in args.extra.split(",")]
+        chosen = EXTRA if args.extra is None else [int(i) for i in args.extra.split(",") if i]
         for idx in chosen:
             we = I.WORKLOADS[idx]
             _, mse, te, nle, pe = bench_workload(we, args.steps, args.warmup)
