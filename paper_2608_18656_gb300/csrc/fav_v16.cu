@@ -12,28 +12,51 @@ namespace {
 // Pass 1: per KV head, the largest finite |v| (as float bits: non-negative floats order like
 // their bit patterns, so an unsigned atomicMax finds it).
 // V rows are read through its strides (element offsets of head (b, g): b * vs.b + g * vs.h,
-// row n: + n * vs.n), D / 8 16-byte chunks per row.
-__device__ __forceinline__ const uint4 *fav_v_chunk(const uint16_t *v, FavStrides vs, int Hkv,
-                                                    long long head, long long i, int d8) {
-    const long long b = head / Hkv, g = head % Hkv, n = i / d8, c = i % d8;
-    return reinterpret_cast<const uint4 *>(v + b * vs.b + g * vs.h + n * vs.n + c * 8);
+// row n: + n * vs.n), D / 8 16-byte chunks per row.  The head's first element is computed once
+// per thread; chunk i of the head is 8 i elements further when its rows are contiguous
+// (vs.n == D), else row i / d8, chunk i % d8 (32-bit arithmetic: i < 2^31).  (64-bit divisions
+// per chunk had left these passes bound by integer arithmetic.)
+__device__ __forceinline__ const uint16_t *fav_v_head(const uint16_t *v, FavStrides vs, int Hkv,
+                                                      long long head) {
+    return v + (head / Hkv) * vs.b + (head % Hkv) * vs.h;
 }
+__device__ __forceinline__ const uint4 *fav_v_chunk(const uint16_t *vh, long long row_stride,
+                                                    bool dense, uint32_t i, uint32_t d8) {
+    if (dense) return reinterpret_cast<const uint4 *>(vh) + i;
+    return reinterpret_cast<const uint4 *>(vh + (long long)(i / d8) * row_stride + (i % d8) * 8);
+}
+
+// Each thread keeps kLoads independent 16-byte loads in flight (chunks i, i + stride, ...):
+// one load per iteration left the passes bound by load latency (1.6 TB/s).
+constexpr int kLoads = 4;
 
 __global__ void __launch_bounds__(256)
 fav_vmax_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
                 unsigned *__restrict__ vmax_bits, long long per_head) {
     const long long head = blockIdx.y;
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    const uint16_t *vh = fav_v_head(v, vs, Hkv, head);
+    const bool dense = vs.n == 8LL * d8;
     unsigned mx = 0;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_head;
-         i += (long long)gridDim.x * blockDim.x) {
-        const uint4 w = *fav_v_chunk(v, vs, Hkv, head, i, d8);
-        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+    for (long long i0 = blockIdx.x * (long long)blockDim.x + threadIdx.x; i0 < per_head;
+         i0 += kLoads * stride) {
+        uint4 w[kLoads];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            // two bf16 values: |x| bits are the low 15 bits of each half, moved to float bits
-            const uint32_t lo = (u[k] & 0x7FFFu) << 16, hi = u[k] & 0x7FFF0000u;
-            if (lo < 0x7F800000u) mx = max(mx, lo);      // finite only
-            if (hi < 0x7F800000u) mx = max(mx, hi);
+        for (int r = 0; r < kLoads; ++r) {
+            const long long i = i0 + r * stride;
+            w[r] = i < per_head ? *fav_v_chunk(vh, vs.n, dense, (uint32_t)i, (uint32_t)d8)
+                                : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int r = 0; r < kLoads; ++r) {
+            const uint32_t u[4] = {w[r].x, w[r].y, w[r].z, w[r].w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                // two bf16 values: |x| bits are the low 15 bits of each half, moved to float bits
+                const uint32_t lo = (u[k] & 0x7FFFu) << 16, hi = u[k] & 0x7FFF0000u;
+                if (lo < 0x7F800000u) mx = max(mx, lo);      // finite only
+                if (hi < 0x7F800000u) mx = max(mx, hi);
+            }
         }
     }
 #pragma unroll
@@ -63,18 +86,32 @@ fav_v16_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
     if (blockIdx.x == 0 && threadIdx.x == 0) v_scale[head] = ldexpf(1.f, e);
     const float inv = ldexpf(1.f, -e);
     uint4 *dst = v16 + head * per_head;        // contiguous [B, Hkv, Nkv, D]
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_head;
-         i += (long long)gridDim.x * blockDim.x) {
-        const uint4 w = *fav_v_chunk(v, vs, Hkv, head, i, d8);
-        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
-        uint32_t r[4];
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    const uint16_t *vh = fav_v_head(v, vs, Hkv, head);
+    const bool dense = vs.n == 8LL * d8;
+    for (long long i0 = blockIdx.x * (long long)blockDim.x + threadIdx.x; i0 < per_head;
+         i0 += kLoads * stride) {
+        uint4 w[kLoads];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const float lo = __uint_as_float(u[k] << 16) * inv;
-            const float hi = __uint_as_float(u[k] & 0xFFFF0000u) * inv;
-            r[k] = fav::Elem<__half>::pack(lo, hi);
+        for (int r = 0; r < kLoads; ++r) {
+            const long long i = i0 + r * stride;
+            w[r] = i < per_head ? *fav_v_chunk(vh, vs.n, dense, (uint32_t)i, (uint32_t)d8)
+                                : make_uint4(0, 0, 0, 0);
         }
-        dst[i] = make_uint4(r[0], r[1], r[2], r[3]);
+#pragma unroll
+        for (int r = 0; r < kLoads; ++r) {
+            const long long i = i0 + r * stride;
+            if (i >= per_head) break;
+            const uint32_t u[4] = {w[r].x, w[r].y, w[r].z, w[r].w};
+            uint32_t h[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float lo = __uint_as_float(u[k] << 16) * inv;
+                const float hi = __uint_as_float(u[k] & 0xFFFF0000u) * inv;
+                h[k] = fav::Elem<__half>::pack(lo, hi);
+            }
+            dst[i] = make_uint4(h[0], h[1], h[2], h[3]);
+        }
     }
 }
 
@@ -105,16 +142,19 @@ fav_status fav_v16_convert(const FavArgs &a, void *workspace, cudaStream_t strea
     float *vsc = reinterpret_cast<float *>(ws + L.scale);
     const long long heads = (long long)a.B * a.Hkv;
     const long long per_head = (long long)a.Nkv * a.D / 8;      // uint4 chunks (D % 8 == 0)
-    if (heads > 65535) return FAV_ERR_UNSUPPORTED;
-    const unsigned bx = (unsigned)std::max<long long>(
-        1, std::min<long long>((per_head + 255) / 256, std::max<long long>(1, 4LL * a.num_sms / heads)));
+    if (heads > 65535 || per_head >= (1LL << 31)) return FAV_ERR_UNSUPPORTED;
     if (cudaMemsetAsync(vmax, 0, heads * sizeof(unsigned), stream) != cudaSuccess)
         return FAV_ERR_CUDA;
-    fav_vmax_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(
-        static_cast<const uint16_t *>(a.v), a.vs, a.Hkv, D / 8, vmax, per_head);
-    fav_v16_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(
-        static_cast<const uint16_t *>(a.v), a.vs, a.Hkv, D / 8,
-        reinterpret_cast<uint4 *>(ws + L.v16), vmax, vsc, per_head);
+    const uint16_t *vsrc = static_cast<const uint16_t *>(a.v);
+    uint4 *v16p = reinterpret_cast<uint4 *>(ws + L.v16);
+    // about eight 256-thread blocks per SM over all heads, each thread with kLoads loads in flight
+    const unsigned bx = (unsigned)std::max<long long>(
+        1, std::min<long long>((per_head + 256LL * kLoads - 1) / (256LL * kLoads),
+                               std::max<long long>(1, 8LL * std::max(1, a.num_sms) / heads)));
+    fav_vmax_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(vsrc, a.vs, a.Hkv, D / 8, vmax,
+                                                                   per_head);
+    fav_v16_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(vsrc, a.vs, a.Hkv, D / 8, v16p,
+                                                                  vmax, vsc, per_head);
     if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_v16_kernel", stream))
         return FAV_ERR_CUDA;
     *v16 = ws + L.v16;
