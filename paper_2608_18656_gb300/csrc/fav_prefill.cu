@@ -122,7 +122,7 @@ template <int D> struct PrefillCfg {
     static constexpr int kXchBytes = 2 * 4 * kSplits * 32 * 8;
     static constexpr int kOffUnits = kOffXch + kXchBytes;         // int[kUnitTab][12]
     static constexpr int kOffBar = kOffUnits + kUnitTab * 48;
-    static constexpr int kNumBars = 2 + 2 + 2 * kKStages + 2 * kVStages + 2 + 2 + 2 + 2 + 2 + 1;
+    static constexpr int kNumBars = 2 + 2 + 2 * kKStages + 2 * kVStages + 2 + 2 + 2 + 2 + 2 + 1 + 2;
     static constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
     static constexpr int kOffDbg = kOffTmemSlot + 16;             // debug builds: per-role totals
     static constexpr int kSmemBytes = kOffDbg + 32 + 1024;
@@ -159,7 +159,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     const uint32_t sQ = sbase + C::kOffQ, sK = sbase + C::kOffK, sV = sbase + C::kOffV;
     const uint32_t bar0 = sbase + C::kOffBar;
     const uint32_t q_full = bar0;                 // [2] per Q buffer
-    const uint32_t q_empty = q_full + 16;         // [2] the buffer's last S read and O stored
+    const uint32_t q_empty = q_full + 16;         // [2] the buffer's last S read (and O stored)
     const uint32_t k_full = q_empty + 16, k_empty = k_full + 8 * KS;
     const uint32_t v_full = k_empty + 8 * KS, v_empty = v_full + 8 * VS;
     const uint32_t s_full = v_empty + 8 * VS;     // [2] per score buffer
@@ -169,6 +169,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
     const uint32_t xch_bar = o_done + 8;          // [2] (m, l) of every row and split written
     const uint32_t o_staged = xch_bar + 16;       // [2] O tile written into Q buffer k % 2
     const uint32_t o_free = o_staged + 16;        // the epilogue has read the unit's O
+    const uint32_t xch_free = o_free + 8;         // [2] the epilogue has read (m, l) slot k % 2
     float2 *xch = reinterpret_cast<float2 *>(smem + C::kOffXch);
     int *utab = reinterpret_cast<int *>(smem + C::kOffUnits);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffTmemSlot);
@@ -296,7 +297,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         (void)FAV_CHECK((sbase - raw_u32) + C::kOffTmemSlot + 4 <= fav::dynamic_smem_bytes(), status);
         for (int i = 0; i < 2; ++i) {
             fav::mbar_init(q_full + 8 * i, 1);
-            fav::mbar_init(q_empty + 8 * i, 2);          // last S commit + O store read
+            // last S commit, + the O store's read of the buffer when O is staged there
+            fav::mbar_init(q_empty + 8 * i, varlen ? 1 : 2);
+            fav::mbar_init(xch_free + 8 * i, 128);          // epilogue threads
             fav::mbar_init(o_staged + 8 * i, 128);          // epilogue threads
             fav::mbar_init(xch_bar + 8 * i, C::kSoftWarps * 32);
             fav::mbar_init(s_full + 8 * i, 1);
@@ -475,7 +478,14 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 if (lane == 0) fav::mbar_arrive(p_full + 8 * (Gt & 1));
             }
             if (!ok) break;
-            // (m, l) of this row and split for the epilogue warpgroup (slot k % 2)
+            // (m, l) of this row and split for the epilogue warpgroup (slot k % 2).  Packed
+            // batches release a Q buffer with its unit's last S (O is not staged there), so unit
+            // k + 2 can reach this point before the epilogue has read unit k's slot: wait for it.
+            if constexpr (varlen) {
+                if (k >= 2 && !__all_sync(~0u, fav::mbar_wait_il(xch_free + 8 * (k & 1),
+                                                                ((k >> 1) - 1) & 1, status)))
+                    break;
+            }
             xch[((((k & 1) * 4 + quarter) * NS) + split) * 32 + lane] = make_float2(m, l);
             fav::mbar_arrive(xch_bar + 8 * (k & 1));
         }
@@ -502,6 +512,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             fav::tc::fence_after();
             const float2 ml0 = xch[((((k & 1) * 4 + quarter) * NS) + 0) * 32 + lane];
             const float2 ml1 = xch[((((k & 1) * 4 + quarter) * NS) + 1) * 32 + lane];
+            if constexpr (varlen) fav::mbar_arrive(xch_free + 8 * (k & 1));
             const float Mx = fmaxf(ml0.x, ml1.x);
             const float w0 = (ml0.x == -INFINITY) ? 0.f : fav::fast_exp2(ml0.x - Mx);
             const float w1 = (ml1.x == -INFINITY) ? 0.f : fav::fast_exp2(ml1.x - Mx);
@@ -511,9 +522,11 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             const float inv_l = vsc / L;
             const float a0 = w0 * inv_l, a1 = w1 * inv_l;
             const uint32_t stage = sQ + (k & 1) * C::kQBytes + row * 128;
-            // the last tile of a packed sequence is written row by row (its rows past the end
-            // belong to the next sequence); every other tile goes through the TMA store
-            const bool partial = varlen && U.t * BM + BM > U.len_q;
+            // Dense calls: the tile goes through the Q buffer and one TMA store.  Packed batches:
+            // every row is written straight to the output (a sequence's last tile has rows of the
+            // next sequence past its end, and the Q buffer is released with the unit's last S, so
+            // short units do not wait on the O store to load the next-but-one Q tile).
+            const bool direct = varlen;
             const bool valid = qi < U.len_q;
             T *orow = o + U.b * os.b + U.h * os.h + (long long)(U.q_y0 + qi) * os.n;
 #pragma unroll
@@ -523,6 +536,11 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                 fav::tc::ld_32x32b_x32(trow + C::kColO + D + c * 32, v1);
                 fav::tc::wait_ld_dep(v0);
                 fav::tc::wait_ld_dep(v1);
+                if (c + 1 == D / 32) {
+                    // O has been read: release it to the next unit's first P.V
+                    fav::tc::fence_before();
+                    fav::mbar_arrive(o_free);
+                }
 #pragma unroll
                 for (int h = 0; h < 4; ++h) {
                     // 8 columns = one 16-byte chunk: column block c / 2, chunk 4 (c % 2) + h
@@ -534,7 +552,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                             fmaf(a0, __uint_as_float(v0[i]), a1 * __uint_as_float(v1[i])),
                             fmaf(a0, __uint_as_float(v0[i + 1]), a1 * __uint_as_float(v1[i + 1])));
                     }
-                    if (!partial) {
+                    if (!direct) {
                         const uint32_t chunk = (uint32_t)(4 * (c & 1) + h) ^ (uint32_t)(row & 7);
                         const uint32_t addr = stage + (c >> 1) * (BM * 128) + (chunk << 4);
                         asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};"
@@ -545,11 +563,10 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
                     }
                 }
             }
-            // O has been read: release it to the next unit's first P.V
-            fav::tc::fence_before();
-            fav::mbar_arrive(o_free);
-            fav::tc::fence_proxy_async_smem();   // visible to the TMA store (async proxy)
-            fav::mbar_arrive(o_staged + 8 * (k & 1));
+            if constexpr (!varlen) {
+                fav::tc::fence_proxy_async_smem();   // visible to the TMA store (async proxy)
+                fav::mbar_arrive(o_staged + 8 * (k & 1));
+            }
             if (valid && lse) {
                 // [B, Hq, Nq] (dense) or [Hq, total_q] (packed: Nq = total_q)
                 const long long li = varlen ? (long long)U.h * Nq + U.q_y0 + qi
@@ -635,20 +652,17 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
 #endif
             }
         } else if (warp == C::kStoreWarp) {
-            // ---------------- O tiles: one TMA store per unit from its (free) Q buffer ----------------
-            if (lane == 0) {
+            // ---------------- O tiles (dense calls): one TMA store per unit from its (free) Q buffer ----------------
+            // (packed batches: the epilogue writes O itself)
+            if (!varlen && lane == 0) {
                 fav::tma_prefetch_desc(&tmO);
                 for (int k = 0, u; (u = unit_at(k)) >= 0; ++k) {
                     const Unit U = unit(k);
                     const int qb = k & 1;
                     if (!fav::mbar_wait_il(o_staged + 8 * qb, (k >> 1) & 1, status)) break;
-                    // (a partial tile of a packed sequence was written by the epilogue: rows past
-                    // its end belong to the next sequence)
-                    if (!(varlen && U.t * BM + BM > U.len_q)) {
-                        fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.q_y0 + U.t * BM, 0, U.h, U.b);
-                        fav::bulk_commit_group();
-                        fav::bulk_wait_read_all();     // the buffer may take the next Q tile
-                    }
+                    fav::tma_store_5d(&tmO, sQ + qb * C::kQBytes, 0, U.q_y0 + U.t * BM, 0, U.h, U.b);
+                    fav::bulk_commit_group();
+                    fav::bulk_wait_read_all();     // the buffer may take the next Q tile
                     fav::mbar_arrive(q_empty + 8 * qb);
 #ifdef FAV_DEBUG_CHECKS
                     dbg_tot[6] = k + 1;
@@ -768,7 +782,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
         (void)FAV_CHECK(dbg_tot[0] == tiles && dbg_tot[1] == tiles && dbg_tot[2] == tiles &&
                             dbg_tot[3] == tiles && dbg_tot[4] == tiles && dbg_tot[5] == units &&
-                            dbg_tot[6] == units,
+                            (varlen || dbg_tot[6] == units),
                         status);
     }
 #endif
