@@ -327,6 +327,21 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
         auto wait_all = [&](uint32_t bar, uint32_t parity) {
             return __all_sync(0xffffffffu, fav::mbar_wait(bar, parity, status));
         };
+        // Two barriers tested with one instruction (lane 0: a, if need_a; lane 1: b), then waited
+        // for one by one only if one of them was not complete.  Each test instruction of this warp
+        // costs it about as much as a short burst of MMAs takes to issue (it waits for the warp's
+        // queued MMAs and commits), and the K / V stages are almost always complete by the time
+        // the softmax has released its scores / stored its weights: testing them with those
+        // barriers instead of separately took C3 from 315.5 to 307.2 us.
+        auto wait_two = [&](uint32_t bar_a, uint32_t par_a, bool need_a, uint32_t bar_b,
+                            uint32_t par_b) -> bool {
+            uint32_t tb = bar_b, tp = par_b;
+            bool need = lane == 1;
+            if (lane == 0) { tb = bar_a; tp = par_a; need = need_a; }
+            if (__all_sync(0xffffffffu, !need || fav::mbar_test(tb, tp))) return true;
+            if (need_a && !wait_all(bar_a, par_a)) return false;
+            return wait_all(bar_b, par_b) != 0;
+        };
         auto try_all = [&](uint32_t bar, uint32_t parity) {
             return __all_sync(0xffffffffu, fav::mbar_try(bar, parity));
         };
@@ -377,17 +392,17 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
 #pragma unroll
                     for (int i = 0; i < 2; ++i) {
                         if (j + 1 < U.n_kv_tiles[i]) {
-                            if (!k_ok && !(ok = wait_all(k_full + 8 * st1, ((gj + 1) / S) & 1))) break;
+                            if (!(ok = wait_two(k_full + 8 * st1, ((gj + 1) / S) & 1, !k_ok,
+                                                s_free + 8 * i, (nsi[i] - 1) & 1))) break;
                             k_ok = true;
-                            if (!(ok = wait_all(s_free + 8 * i, (nsi[i] - 1) & 1))) break;
                             fav::tc::fence_after();
                             issue_s(i, st1, s_full + 8 * i, i == last1 ? k_empty + 8 * st1 : 0u);
                             ++nsi[i];
                         }
                         if (j < U.n_kv_tiles[i]) {
-                            if (!v_ok && !(ok = wait_all(v_full + 8 * st, (gj / S) & 1))) break;
+                            if (!(ok = wait_two(v_full + 8 * st, (gj / S) & 1, !v_ok,
+                                                p_full + 8 * i, np[i] & 1))) break;
                             v_ok = true;
-                            if (!(ok = wait_all(p_full + 8 * i, np[i] & 1))) break;
                             ++np[i];
                             fav::tc::fence_after();
                             issue_pv(i, st, j > 0 ? 1u : 0u, p_free + 8 * i, i == last ? v_empty + 8 * st : 0u);
