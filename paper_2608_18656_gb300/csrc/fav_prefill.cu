@@ -518,6 +518,7 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
             const float w1 = (ml1.x == -INFINITY) ? 0.f : fav::fast_exp2(ml1.x - Mx);
             const float L = w0 * ml0.y + w1 * ml1.y;
             const int qi = U.t * BM + row;
+            if constexpr (kV16) asm volatile("griddepcontrol.wait;" ::: "memory");   // v_scale
             const float vsc = kV16 ? v_scale[U.b * Hkv + U.kvh] : 1.f;   // V = v_scale * (fp16 copy)
             const float inv_l = vsc / L;
             const float a0 = w0 * inv_l, a1 = w1 * inv_l;
@@ -629,6 +630,9 @@ fav_prefill_split_kernel(const __grid_constant__ CUtensorMap tmQ,
         } else if (warp == C::kLoadVWarp) {
             // ---------------- TMA producer: V tiles ----------------
             if (lane == 0) {
+                // bf16 I/O: this kernel is a programmatic dependent of the V conversion, whose
+                // output the V copies read (the set-up, Q and K copies go ahead of it)
+                if constexpr (kV16) asm volatile("griddepcontrol.wait;" ::: "memory");
                 fav::tma_prefetch_desc(&tmV);
                 int g = 0;
                 bool ok = true;
@@ -829,10 +833,22 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream,
     groups_per_block = std::min<long long>(groups_per_block, (long long)a.B * a.Hkv);
     int head_block = (int)(groups_per_block * G);
     if ((units + blocks - 1) / blocks > C::kUnitTab) head_block = a.B * a.Hq;
-    kern<<<(unsigned)blocks, C::kThreads, C::kSmemBytes, stream>>>(
-        tmQ, tmK, tmV, tmO, (T *)a.o, a.os, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv,
-        n_qtiles, head_block, a.scale * kLog2e, a.causal, a.dev_status, vunits, n_vunits);
-    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_split_kernel", stream))
+    // bf16 I/O: a programmatic dependent of the V conversion (set-up, Q and K copies overlap its
+    // tail; V and its scales are read after griddepcontrol.wait)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3(C::kThreads);
+    cfg.dynamicSmemBytes = C::kSmemBytes;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = kV16 ? 1 : 0;
+    if (cudaLaunchKernelEx(&cfg, kern, tmQ, tmK, tmV, tmO, (T *)a.o, a.os, a.lse, v_scale, a.B,
+                           a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles, head_block, a.scale * kLog2e,
+                           a.causal, a.dev_status, vunits, n_vunits) != cudaSuccess ||
+        cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_split_kernel", stream))
         return FAV_ERR_CUDA;
     return FAV_OK;
 }

@@ -265,6 +265,9 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
             fav::tma_prefetch_desc(&tmV);
             int g = 0;
             bool ok = true;
+            // bf16 I/O: this kernel is a programmatic dependent of the V conversion, whose output
+            // the V copies read: wait for that grid before the first one (Q and K copies go ahead)
+            bool v_ready = !kV16;
             for (int k = 0, u; ok && (u = unit_at(k)) >= 0; ++k) {
                 const Unit U = make_unit(u);
                 // the Q buffers are free once the previous unit's last S MMA has completed; both
@@ -289,6 +292,10 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
                         fav::tma_load_4d(sK + st * C::kKVBytes + bx * BN * 128, &tmK, k_full + 8 * st,
                                          bx * 64, U.k_y0 + j * BN, U.kvh, U.b);
                     if (g >= S && !fav::mbar_wait(v_empty + 8 * st, ph, status)) { ok = false; break; }
+                    if (!v_ready) {
+                        asm volatile("griddepcontrol.wait;" ::: "memory");
+                        v_ready = true;
+                    }
                     fav::mbar_arrive_expect_tx(v_full + 8 * st, C::kKVBytes);
 #pragma unroll
                     for (int bx = 0; bx < C::kBoxes; ++bx)
@@ -564,6 +571,7 @@ fav_prefill_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_co
             if (!__all_sync(~0u, fav::mbar_wait(o_done + 8 * i, no & 1, status))) { ok = false; break; }
             ++no;
             fav::tc::fence_after();
+            if constexpr (kV16) asm volatile("griddepcontrol.wait;" ::: "memory");   // v_scale
             const float vsc = kV16 ? v_scale[U.bkv] : 1.f;     // V = v_scale * (fp16 copy)
             const float inv_l = vsc / l;
             const bool valid = qi < U.len_q;
@@ -633,10 +641,22 @@ fav_status launch(const FavArgs &a, void *workspace, cudaStream_t stream,
     // persistent: one CTA per SM at most, each working through its share of the units
     long long blocks = std::min<long long>(units, std::max(1, a.num_sms));
     if (a.prefill_grid > 0) blocks = std::min<long long>(blocks, a.prefill_grid);
-    kern<<<(unsigned)blocks, kThreads, C::kSmemBytes, stream>>>(
-        tmQ, tmK, tmV, (T *)a.o, a.os, a.lse, v_scale, a.B, a.Hq, a.Hkv, a.Nq, a.Nkv, n_qtiles,
-        pair_heads, a.scale * kLog2e, a.causal, a.dev_status, vunits, n_vunits);
-    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_pair_kernel", stream))
+    // bf16 I/O: a programmatic dependent of the V conversion (set-up, Q and K copies overlap its
+    // tail; V and its scales are read after griddepcontrol.wait)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::kSmemBytes;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = kV16 ? 1 : 0;
+    if (cudaLaunchKernelEx(&cfg, kern, tmQ, tmK, tmV, (T *)a.o, a.os, a.lse, v_scale, a.B, a.Hq,
+                           a.Hkv, a.Nq, a.Nkv, n_qtiles, pair_heads, a.scale * kLog2e, a.causal,
+                           a.dev_status, vunits, n_vunits) != cudaSuccess ||
+        cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_prefill_pair_kernel", stream))
         return FAV_ERR_CUDA;
     return FAV_OK;
 }

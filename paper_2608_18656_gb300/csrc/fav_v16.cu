@@ -9,8 +9,10 @@
 
 namespace {
 
-// Pass 1: per KV head, the largest finite |v| (as float bits: non-negative floats order like
-// their bit patterns, so an unsigned atomicMax finds it).
+// Pass 1: per KV head and block, the largest finite |v| (as float bits: non-negative floats
+// order like their bit patterns), written to vmax_part[head * gridDim.x + blockIdx.x]; every
+// slot is written, so the array needs no initialisation and no atomics.  The next pass is
+// launched as a programmatic dependent: it may be scheduled once every block here has started.
 // V rows are read through its strides (element offsets of head (b, g): b * vs.b + g * vs.h,
 // row n: + n * vs.n), D / 8 16-byte chunks per row.  The head's first element is computed once
 // per thread; chunk i of the head is 8 i elements further when its rows are contiguous
@@ -32,7 +34,9 @@ constexpr int kLoads = 4;
 
 __global__ void __launch_bounds__(256)
 fav_vmax_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
-                unsigned *__restrict__ vmax_bits, long long per_head) {
+                unsigned *__restrict__ vmax_part, long long per_head) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    __shared__ unsigned wmax[8];
     const long long head = blockIdx.y;
     const long long stride = (long long)gridDim.x * blockDim.x;
     const uint16_t *vh = fav_v_head(v, vs, Hkv, head);
@@ -61,7 +65,13 @@ fav_vmax_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
     }
 #pragma unroll
     for (int d = 16; d > 0; d >>= 1) mx = max(mx, __shfl_xor_sync(~0u, mx, d));
-    if ((threadIdx.x & 31) == 0 && mx) atomicMax(vmax_bits + head, mx);
+    if ((threadIdx.x & 31) == 0) wmax[threadIdx.x >> 5] = mx;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+#pragma unroll
+        for (int w = 1; w < 8; ++w) mx = max(mx, wmax[w]);
+        vmax_part[head * gridDim.x + blockIdx.x] = mx;
+    }
 }
 
 // Scale exponent of a head: e = floor(log2(max|v|)) - 14, so that max|v| * 2^-e < 2^15 (fp16
@@ -76,13 +86,26 @@ __device__ __forceinline__ int fav_v16_exponent(unsigned vmax_bits) {
 // Pass 2: v16 = fp16(v * 2^-e).  A bf16 value has 8 significant bits, which fp16 holds exactly
 // down to 2^-17 (subnormals included), so every |v| >= 2^(e-17) -- everything within about
 // 2^-31 of the head's maximum -- converts exactly; smaller values err by less than 2^(e-25).
-// Non-finite values stay non-finite.  Also stores v_scale = 2^e.
+// Non-finite values stay non-finite.  Also stores v_scale = 2^e.  A programmatic dependent of
+// pass 1 (it waits for that grid's completion before reading the partial maxima); the prefill
+// kernel is in turn launched as a dependent of this one.
 __global__ void __launch_bounds__(256)
 fav_v16_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
-               uint4 *__restrict__ v16, const unsigned *__restrict__ vmax_bits,
+               uint4 *__restrict__ v16, const unsigned *__restrict__ vmax_part,
                float *__restrict__ v_scale, long long per_head) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    __shared__ unsigned head_max;
     const long long head = blockIdx.y;
-    const int e = fav_v16_exponent(vmax_bits[head]);
+    if (threadIdx.x < 32) {   // the head's maximum from pass 1's gridDim.x (= this grid's) partials
+        unsigned m = 0;
+        for (unsigned i = threadIdx.x; i < gridDim.x; i += 32) m = max(m, vmax_part[head * gridDim.x + i]);
+#pragma unroll
+        for (int d = 16; d > 0; d >>= 1) m = max(m, __shfl_xor_sync(~0u, m, d));
+        if (threadIdx.x == 0) head_max = m;
+    }
+    __syncthreads();
+    const int e = fav_v16_exponent(head_max);
     if (blockIdx.x == 0 && threadIdx.x == 0) v_scale[head] = ldexpf(1.f, e);
     const float inv = ldexpf(1.f, -e);
     uint4 *dst = v16 + head * per_head;        // contiguous [B, Hkv, Nkv, D]
@@ -115,7 +138,17 @@ fav_v16_kernel(const uint16_t *__restrict__ v, FavStrides vs, int Hkv, int d8,
     }
 }
 
-// workspace of the kV16 path: [fp16 V][vmax bits per KV head][scale per KV head]
+// Blocks per KV head of both passes: about eight 256-thread blocks per SM over all heads, each
+// thread with kLoads loads in flight.
+unsigned v16_blocks_x(const FavArgs &a) {
+    const long long heads = (long long)a.B * a.Hkv;
+    const long long per_head = (long long)a.Nkv * a.D / 8;      // uint4 chunks (D % 8 == 0)
+    return (unsigned)std::max<long long>(
+        1, std::min<long long>((per_head + 256LL * kLoads - 1) / (256LL * kLoads),
+                               std::max<long long>(1, 8LL * std::max(1, a.num_sms) / std::max(1LL, heads))));
+}
+
+// workspace of the kV16 path: [fp16 V][per-block maxima: heads x blocks][scale per KV head]
 struct V16Layout {
     size_t v16, vmax, scale, total;
     explicit V16Layout(const FavArgs &a) {
@@ -123,7 +156,7 @@ struct V16Layout {
         auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
         v16 = 0;
         vmax = up(heads * a.Nkv * a.D * 2);
-        scale = vmax + up(heads * 4);
+        scale = vmax + up(heads * v16_blocks_x(a) * 4);
         total = scale + up(heads * 4);
     }
 };
@@ -143,19 +176,26 @@ fav_status fav_v16_convert(const FavArgs &a, void *workspace, cudaStream_t strea
     const long long heads = (long long)a.B * a.Hkv;
     const long long per_head = (long long)a.Nkv * a.D / 8;      // uint4 chunks (D % 8 == 0)
     if (heads > 65535 || per_head >= (1LL << 31)) return FAV_ERR_UNSUPPORTED;
-    if (cudaMemsetAsync(vmax, 0, heads * sizeof(unsigned), stream) != cudaSuccess)
-        return FAV_ERR_CUDA;
     const uint16_t *vsrc = static_cast<const uint16_t *>(a.v);
     uint4 *v16p = reinterpret_cast<uint4 *>(ws + L.v16);
-    // about eight 256-thread blocks per SM over all heads, each thread with kLoads loads in flight
-    const unsigned bx = (unsigned)std::max<long long>(
-        1, std::min<long long>((per_head + 256LL * kLoads - 1) / (256LL * kLoads),
-                               std::max<long long>(1, 8LL * std::max(1, a.num_sms) / heads)));
+    const unsigned bx = v16_blocks_x(a);
     fav_vmax_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(vsrc, a.vs, a.Hkv, D / 8, vmax,
                                                                    per_head);
-    fav_v16_kernel<<<dim3(bx, (unsigned)heads), 256, 0, stream>>>(vsrc, a.vs, a.Hkv, D / 8, v16p,
-                                                                  vmax, vsc, per_head);
-    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_v16_kernel", stream))
+    if (cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_vmax_kernel", stream))
+        return FAV_ERR_CUDA;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(bx, (unsigned)heads);
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, fav_v16_kernel, vsrc, a.vs, a.Hkv, D / 8, v16p,
+                           (const unsigned *)vmax, vsc, per_head) != cudaSuccess ||
+        cudaGetLastError() != cudaSuccess || fav_debug_sync("fav_v16_kernel", stream))
         return FAV_ERR_CUDA;
     *v16 = ws + L.v16;
     *v16_strides = fav_contiguous_strides(a.Hkv, a.Nkv, D);
