@@ -424,6 +424,28 @@ fav_combine_kernel(const float *__restrict__ part_o, const float *__restrict__ p
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (row >= rows) return;
     const float *pl = part_lse + row * splits;
+    // Each warp's first two splits of O are requested together with the LSE partials (one round
+    // trip to L2 instead of two on the call's critical path).
+    constexpr int kPer = D / 32;                  // consecutive columns per lane
+    const float *po = part_o + row * splits * D + lane * kPer;
+    float pre[2][kPer];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        const int sp = warp + 4 * r;
+        if (sp < splits) {
+            const float *src = po + (long long)sp * D;
+            if constexpr (kPer == 4) {
+                const float4 x = *reinterpret_cast<const float4 *>(src);
+                pre[r][0] = x.x; pre[r][1] = x.y; pre[r][2] = x.z; pre[r][3] = x.w;
+            } else {
+                const float2 x = *reinterpret_cast<const float2 *>(src);
+                pre[r][0] = x.x; pre[r][1] = x.y;
+            }
+        } else {
+#pragma unroll
+            for (int c = 0; c < kPer; ++c) pre[r][c] = 0.f;
+        }
+    }
     float mx = -INFINITY;
     for (int s = threadIdx.x; s < splits; s += 128) mx = fmaxf(mx, pl[s]);
 #pragma unroll
@@ -440,13 +462,21 @@ fav_combine_kernel(const float *__restrict__ part_o, const float *__restrict__ p
     if (lane == 0) wred[warp] = sum;
     __syncthreads();
     const float L = mx + logf(wred[0] + wred[1] + wred[2] + wred[3]);
-    constexpr int kPer = D / 32;                  // consecutive columns per lane
     float acc[kPer];
 #pragma unroll
     for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
-    const float *po = part_o + row * splits * D + lane * kPer;
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        const int sp = warp + 4 * r;
+        if (sp < splits) {
+            const float ls = pl[sp];
+            const float w = (ls == -INFINITY) ? 0.f : expf(ls - L);
+#pragma unroll
+            for (int c = 0; c < kPer; ++c) acc[c] = fmaf(w, pre[r][c], acc[c]);
+        }
+    }
 #pragma unroll 4
-    for (int s = warp; s < splits; s += 4) {
+    for (int s = warp + 8; s < splits; s += 4) {
         const float ls = pl[s];
         const float w = (ls == -INFINITY) ? 0.f : expf(ls - L);
         const float *src = po + (long long)s * D;
