@@ -6,7 +6,9 @@ a process that waits on and arrives at mbarriers exactly as the kernel source do
 per-CTA unit lists (snake order, heaviest query tile first), the same stage indices and phase
 parities, arrival counts, expected transaction bytes and tcgen05 commits.  TMA copies and MMA
 bursts complete after random delays and the processes run in random order.  A run must finish
-with no process left waiting and no barrier receiving more arrivals than its count in a phase;
+with no process left waiting and no barrier receiving more arrivals than its count in a phase
+(also in the packed-batch variant: O rows written by the epilogue, Q buffers released by the last
+S, back-pressure on the (m, l) exchange slots, whose removal the model catches);
 every parity wait must pass exactly when the phase it stands for has completed (not before it,
 and not after a later phase of the same barrier); a deliberately wrong parity must be caught.  (The GPU tests check the results; this checks
 the orderings that a GPU run only samples.)
@@ -64,10 +66,13 @@ def units_of(B, Hq, Nq, Nkv, P, c, causal=True):
         k += 1
 
 
-def simulate(units, rng, mistake=None):
+def simulate(units, rng, mistake=None, packed=False):
+    """packed: the packed-batch variant (the epilogue writes O rows itself, so a Q buffer is
+    released by its unit's last S alone, and the (m, l) exchange slot k % 2 has a back-pressure
+    barrier: the softmax waits for the epilogue to have read unit k - 2's slot)."""
     bars = {}
-    for name, count in [("q_full", 1), ("q_empty", 2), ("o_staged", 128), ("xch_bar", 256),
-                        ("s_full", 1), ("p_full", 8)]:
+    for name, count in [("q_full", 1), ("q_empty", 1 if packed else 2), ("o_staged", 128),
+                        ("xch_bar", 256), ("xch_free", 128), ("s_full", 1), ("p_full", 8)]:
         for i in range(2):
             bars["%s%d" % (name, i)] = Bar("%s%d" % (name, i), count)
     for i in range(KS):
@@ -180,6 +185,8 @@ def simulate(units, rng, mistake=None):
                 bars["p_full%d" % (Gt & 1)].arrive()
                 Gt += 1
                 yield None
+            if packed and packed != "no_backpressure" and k >= 2:   # unit k - 2's (m, l) read
+                yield ("wait", "xch_free%d" % (k & 1), (k >> 1) - 1)
             bars["xch_bar%d" % (k & 1)].arrive(32)
             yield None
 
@@ -187,12 +194,23 @@ def simulate(units, rng, mistake=None):
         for k in range(n):
             yield ("wait", "o_done", k)
             yield ("wait", "xch_bar%d" % (k & 1), k >> 1)
+            if packed:                             # (m, l) read: the slot is free again
+                bars["xch_free%d" % (k & 1)].arrive(32)
+                yield None
             bars["o_free"].arrive(32)
             yield None
-            bars["o_staged%d" % (k & 1)].arrive(32)
-            yield None
+            if packed:                             # the O rows' stores to global memory take a while
+                stored = [False]
+                at(now[0] + rng.uniform(0.1, 4.0), lambda: stored.__setitem__(0, True))
+                yield ("until", stored)
+            if not packed:                         # O staged for the store warp's TMA store
+                bars["o_staged%d" % (k & 1)].arrive(32)
+                yield None
 
     def store_warp():
+        if packed:                                 # the epilogue writes O itself
+            return
+            yield
         for k in range(n):
             yield ("wait", "o_staged%d" % (k & 1), k >> 1)
             read = [False]
@@ -283,12 +301,32 @@ def test_planted_parity_mistake_is_caught():
             assert stuck and stuck["mma"][1].startswith("q_full")
 
 
-def test_protocol_packed_batch_unit_mixes():
+@pytest.mark.parametrize("packed", [False, True])
+def test_protocol_packed_batch_unit_mixes(packed):
     """A packed variable-length batch gives a block units of any key-tile count (sequences of
-    different lengths, ragged last tiles) in the host's heaviest-first order."""
+    different lengths, ragged last tiles) in the host's heaviest-first order; run with the dense
+    kernel's O staging and with the packed variant's own protocol (direct O rows, Q buffer
+    released by the last S, back-pressure on the (m, l) exchange slots)."""
     rng = random.Random(18656)
     for _ in range(60):
         units = [{"t": 0, "n_kv": rng.randint(1, 10)} for _ in range(rng.randint(1, 12))]
         units.sort(key=lambda U: -U["n_kv"])
-        stuck = simulate(units, random.Random(rng.random()))
+        stuck = simulate(units, random.Random(rng.random()), packed=packed)
         assert not stuck, (units, stuck)
+
+
+def test_packed_exchange_without_back_pressure_is_caught():
+    """Planted in the model: the packed variant without the exchange slot's back-pressure wait
+    lets the softmax complete a second phase of xch_bar (unit k + 2) before the epilogue has
+    waited for the first (unit k): the epilogue then either passes a later phase (the exact-phase
+    check) or never sees its phase (left waiting), on units of one key tile."""
+    units = [{"t": 0, "n_kv": 1} for _ in range(8)]
+    caught = 0
+    for trial in range(40):
+        try:
+            stuck = simulate(units, random.Random(trial), packed="no_backpressure")
+        except AssertionError as e:
+            caught += "xch_bar" in str(e) or "more arrivals" in str(e)
+        else:
+            caught += any(w and w[0] == "wait" and w[1].startswith("xch_bar") for w in stuck.values())
+    assert caught > 0
