@@ -49,5 +49,7 @@ def test_kernel_hash_ignores_comments_but_not_code(tmp_path, monkeypatch):
     text = f.read_text()
     f.write_text("// a new comment line\n/* and a block\n   comment */\n" + text + "\n\n")
     assert bench.kernel_hash() == h0
-    f.write_text(text.replace("kPrefetch = 4", "kPrefetch = 3", 1))
+    changed = text.replace("kRescaleThreshold = 4.0f", "kRescaleThreshold = 3.0f", 1)
+    assert changed != text                  # the constant this test edits still exists
+    f.write_text(changed)
     assert bench.kernel_hash() != h0
